@@ -1,0 +1,184 @@
+"""CPU oracle for top-k attention -- TEST INFRASTRUCTURE ONLY.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the ``cpu_baseline`` /
+``--impl reference`` legs of ``bench.py`` may import this package.  The
+product path (``paper_2106_06899_gb300``) never imports, links or runs it.
+
+It wraps ``topk_oracle.c`` (plain C, fp64, one pthread per host core), which
+computes the paper's definitions directly:
+
+* Eq. 4 -- top-k attention: keep the k largest scores of each row of Q K^T,
+  softmax over those k only, weighted sum of the matching value rows;
+* Eq. 3 -- the feed-forward layer cast as attention: Q = x, K = W1, V = W2,
+  ReLU in place of softmax;
+* Eq. 1 / Eq. 2 -- plain (optionally causal) attention over every key, the
+  special case top-k reduces to when k equals the number of keys;
+* index-evaluate mode: the same activation and weighted sum for a given
+  kept set (used where the near-tie rule lets two correct sets differ).
+
+Ties are broken toward the lower key index; causal rows with fewer than k
+valid keys keep all of them.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "topk_oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+F32, BF16 = 0, 1
+SOFTMAX, RELU = 0, 1
+
+
+def build(force: bool = False) -> str:
+    """Compile topk_oracle.c into liboracle.so (gcc -O2, no fast-math)."""
+    if force or not os.path.exists(_LIB) or os.path.getmtime(_LIB) < os.path.getmtime(_SRC):
+        tmp = _LIB + f".tmp{os.getpid()}"
+        subprocess.run(
+            ["gcc", "-O2", "-std=c11", "-D_POSIX_C_SOURCE=200809L", "-shared", "-fPIC", "-pthread",
+             "-o", tmp, _SRC, "-lm"],
+            check=True,
+        )
+        os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            build()
+            lib = ctypes.CDLL(_LIB)
+            i64, i32, vp = ctypes.c_int64, ctypes.c_int, ctypes.c_void_p
+            lib.oracle_topk.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i64, i32, vp, i64,
+                                        vp, vp, vp, vp, i32]
+            lib.oracle_vanilla.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i32, vp, i64, vp, i32]
+            lib.oracle_eval_indices.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i64, vp, i64,
+                                                vp, vp, vp, i32]
+            lib.oracle_hardware_threads.argtypes = []
+            for f in (lib.oracle_topk, lib.oracle_vanilla, lib.oracle_eval_indices, lib.oracle_hardware_threads):
+                f.restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def hardware_threads() -> int:
+    return int(_load().oracle_hardware_threads())
+
+
+def _as_raw(a):
+    """numpy float32 / uint16(bf16 bits) array, or a CPU torch tensor -> (contiguous ndarray, dtype code)."""
+    if not isinstance(a, np.ndarray):  # torch tensor
+        import torch
+
+        t = a.detach().cpu().contiguous()
+        if t.dtype == torch.bfloat16:
+            return t.view(torch.int16).numpy().view(np.uint16), BF16
+        if t.dtype == torch.float32:
+            return t.numpy(), F32
+        raise TypeError(f"oracle takes float32 or bfloat16, got {t.dtype}")
+    a = np.ascontiguousarray(a)
+    if a.dtype == np.float32:
+        return a, F32
+    if a.dtype == np.uint16:
+        return a, BF16
+    raise TypeError(f"oracle takes float32 or bf16-as-uint16 arrays, got {a.dtype}")
+
+
+def _rows_arg(rows, total):
+    if rows is None:
+        return None, total, None
+    r = np.ascontiguousarray(np.asarray(rows, dtype=np.int64))
+    if r.size and (r.min() < 0 or r.max() >= total):
+        raise ValueError("row index out of range")
+    return r, r.size, r.ctypes.data
+
+
+def _common(q, k, v, act):
+    qa, dt = _as_raw(q)
+    ka, dt2 = _as_raw(k)
+    va, dt3 = _as_raw(v)
+    if not (dt == dt2 == dt3):
+        raise TypeError("q, k, v must share a dtype")
+    return qa, ka, va, dt
+
+
+def topk_attention(q, k, v, topk: int, *, act: int = SOFTMAX, causal: bool = False, rows=None, threads: int = 0):
+    """Eq. 4 (act=SOFTMAX) or Eq. 3 (act=RELU) for q [B,H,Lq,d], k/v [B,H,Lk,d].
+
+    Returns dict(out [n,d] f64, idx [n,topk] i32 (-1 pad), score [n,topk] f64 (-inf pad),
+    next_score [n] f64 (the (k+1)-th score, -inf if none)); n = len(rows) or B*H*Lq.
+    """
+    qa, ka, va, dt = _common(q, k, v, act)
+    B, H, Lq, d = qa.shape
+    Lk = ka.shape[2]
+    if ka.shape != (B, H, Lk, d) or va.shape != (B, H, Lk, d):
+        raise ValueError("shape mismatch")
+    r, n, rp = _rows_arg(rows, B * H * Lq)
+    out = np.zeros((n, d), np.float64)
+    idx = np.zeros((n, topk), np.int32)
+    score = np.zeros((n, topk), np.float64)
+    nxt = np.zeros((n,), np.float64)
+    rc = _load().oracle_topk(act, dt, qa.ctypes.data, ka.ctypes.data, va.ctypes.data, B, H, Lq, Lk, d, topk,
+                             int(causal), rp, n, out.ctypes.data, idx.ctypes.data, score.ctypes.data,
+                             nxt.ctypes.data, threads)
+    if rc:
+        raise RuntimeError(f"oracle_topk failed: {rc}")
+    return {"out": out, "idx": idx, "score": score, "next_score": nxt}
+
+
+def vanilla(q, k, v, *, act: int = SOFTMAX, causal: bool = False, rows=None, threads: int = 0):
+    """Eq. 1 (softmax over all valid keys; causal mask of Eq. 2) -> out [n, d] f64."""
+    qa, ka, va, dt = _common(q, k, v, act)
+    B, H, Lq, d = qa.shape
+    Lk = ka.shape[2]
+    r, n, rp = _rows_arg(rows, B * H * Lq)
+    out = np.zeros((n, d), np.float64)
+    rc = _load().oracle_vanilla(act, dt, qa.ctypes.data, ka.ctypes.data, va.ctypes.data, B, H, Lq, Lk, d,
+                                int(causal), rp, n, out.ctypes.data, threads)
+    if rc:
+        raise RuntimeError(f"oracle_vanilla failed: {rc}")
+    return out
+
+
+def eval_indices(q, k, v, idx, *, act: int = SOFTMAX, rows=None, threads: int = 0):
+    """Index-evaluate: given kept sets idx [n, topk] (-1 = empty), return (out [n,d], score [n,topk])."""
+    qa, ka, va, dt = _common(q, k, v, act)
+    B, H, Lq, d = qa.shape
+    Lk = ka.shape[2]
+    r, n, rp = _rows_arg(rows, B * H * Lq)
+    ia = np.ascontiguousarray(np.asarray(idx, dtype=np.int32))
+    if ia.shape[0] != n:
+        raise ValueError("idx rows must match the listed rows")
+    K = ia.shape[1]
+    out = np.zeros((n, d), np.float64)
+    score = np.zeros((n, K), np.float64)
+    rc = _load().oracle_eval_indices(act, dt, qa.ctypes.data, ka.ctypes.data, va.ctypes.data, B, H, Lq, Lk, d,
+                                     K, rp, n, ia.ctypes.data, out.ctypes.data, score.ctypes.data, threads)
+    if rc:
+        raise RuntimeError(f"oracle_eval_indices failed: {rc}")
+    return out, score
+
+
+def ffn(x, W1, W2, topk: int, *, rows=None, threads: int = 0):
+    """Eq. 3 with top-k: x [N, dm], W1/W2 [d_ff, dm] -> same dict as topk()."""
+    return topk_attention(x[None, None], W1[None, None], W2[None, None], topk, act=RELU, rows=rows,
+                             threads=threads)
+
+
+def ffn_dense(x, W1, W2, *, rows=None, threads: int = 0):
+    """Eq. 3 without top-k: ReLU(x W1^T) W2 over every key -> [n, dm] f64."""
+    return vanilla(x[None, None], W1[None, None], W2[None, None], act=RELU, rows=rows, threads=threads)
+
+
+def ffn_eval_indices(x, W1, W2, idx, *, rows=None, threads: int = 0):
+    return eval_indices(x[None, None], W1[None, None], W2[None, None], idx, act=RELU, rows=rows,
+                        threads=threads)

@@ -1,0 +1,334 @@
+/*
+ * topk_oracle.c -- plain, slow, fp64 CPU oracle for top-k attention.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path may link, load or
+ * call this file; only the tests, the package's smoke check and the CPU
+ * baseline leg of the benchmark do.  It shares no code, header, table or
+ * helper with the CUDA library.
+ *
+ * What it computes, per query row i of problem (b, h), written out from the
+ * paper's definitions with no blocking, fusion or reordering:
+ *
+ *   Eq. 1  (dot-product attention, temperature folded into Q):
+ *            s_ij = sum_t q_i[t] * k_j[t]
+ *   Eq. 2  (masking): with the causal mask only keys j <= i are valid.
+ *   Eq. 4  (top-k attention): keep the k largest s_ij of row i, apply the
+ *            activation to those k entries only, and weight the value rows:
+ *            out_i = sum_{j in topk(i)} act(s_i, topk(i))_j * v_j
+ *          act = softmax over the kept entries (attention), or
+ *   Eq. 3  act = ReLU applied entry-wise (feed-forward layer cast as
+ *          attention: Q = x, K = W1, V = W2, rows of W1/W2 are keys/values).
+ *
+ * Readings where the paper is silent (Sec. 2.2 gives none of these):
+ *   - ties in s are broken toward the lower key index, i.e. the kept set is
+ *     the first k entries of the total order (s descending, j ascending);
+ *   - a causal row with fewer than k valid keys keeps all of them
+ *     (k_eff = i + 1), and the softmax covers those only;
+ *   - top-k runs on the signed scores; ReLU is applied after selection.
+ *
+ * Arithmetic: inputs are widened exactly to double (bf16 by a 16-bit
+ * shift); all sums, the softmax and the weighted sum are in double.
+ * Selection keeps a bounded heap of the k+1 best entries so that the
+ * (k+1)-th score, which decides the near-tie rule, is reported too.
+ */
+#include <math.h>
+#include <pthread.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#include <unistd.h>
+
+#define ORACLE_F32 0
+#define ORACLE_BF16 1
+#define ACT_SOFTMAX 0
+#define ACT_RELU 1
+
+static double widen(const void* base, size_t i, int dtype) {
+  if (dtype == ORACLE_F32) return (double)((const float*)base)[i];
+  uint32_t bits = ((uint32_t)((const uint16_t*)base)[i]) << 16;
+  float f;
+  memcpy(&f, &bits, sizeof f);
+  return (double)f;
+}
+
+typedef struct {
+  double s;
+  int32_t j;
+} entry;
+
+/* a ranks below b in the total order (s descending, j ascending) */
+static int ranks_below(entry a, entry b) {
+  return a.s < b.s || (a.s == b.s && a.j > b.j);
+}
+
+/* Min-heap keyed by rank: h[0] is the lowest-ranked entry kept. */
+static void heap_sift_down(entry* h, int n, int p) {
+  for (;;) {
+    int c = 2 * p + 1;
+    if (c >= n) return;
+    if (c + 1 < n && ranks_below(h[c + 1], h[c])) c++;
+    if (!ranks_below(h[c], h[p])) return;
+    entry t = h[c];
+    h[c] = h[p];
+    h[p] = t;
+    p = c;
+  }
+}
+
+static void heap_sift_up(entry* h, int c) {
+  while (c > 0) {
+    int p = (c - 1) / 2;
+    if (!ranks_below(h[c], h[p])) return;
+    entry t = h[c];
+    h[c] = h[p];
+    h[p] = t;
+    c = p;
+  }
+}
+
+static int cmp_rank_desc(const void* a, const void* b) {
+  const entry* x = (const entry*)a;
+  const entry* y = (const entry*)b;
+  if (ranks_below(*y, *x)) return -1;
+  if (ranks_below(*x, *y)) return 1;
+  return 0;
+}
+
+typedef struct {
+  int act, dtype;
+  const void *q, *k, *v;
+  int64_t H, Lq, Lk, d, topk;
+  int causal, vanilla;
+  const int64_t* rows;
+  int64_t nrows;
+  const int32_t* eval_idx; /* index-evaluate mode when non-NULL */
+  double *out, *score, *next_score;
+  int32_t* idx;
+  int64_t begin, end;
+  int status;
+} job;
+
+static double dot_row(const job* J, int64_t krow, const double* qbuf) {
+  double acc = 0.0;
+  for (int64_t t = 0; t < J->d; ++t) acc += qbuf[t] * widen(J->k, (size_t)(krow * J->d + t), J->dtype);
+  return acc;
+}
+
+static void* run_rows(void* arg) {
+  job* J = (job*)arg;
+  const int64_t d = J->d, K = J->topk;
+  double* qbuf = (double*)malloc(sizeof(double) * (size_t)d);
+  entry* heap = (entry*)malloc(sizeof(entry) * (size_t)(K + 1 > 1 ? K + 1 : 1));
+  entry* sel = (entry*)malloc(sizeof(entry) * (size_t)(J->Lk > K + 1 ? J->Lk : K + 1));
+  double* w = (double*)malloc(sizeof(double) * (size_t)(J->Lk > K ? J->Lk : K));
+  if (!qbuf || !heap || !sel || !w) {
+    J->status = -1;
+    goto done;
+  }
+  for (int64_t r = J->begin; r < J->end; ++r) {
+    const int64_t row = J->rows ? J->rows[r] : r;
+    const int64_t bh = row / J->Lq, i = row % J->Lq;
+    for (int64_t t = 0; t < d; ++t) qbuf[t] = widen(J->q, (size_t)(row * d + t), J->dtype);
+    const int64_t nvalid = J->causal ? (i + 1 < J->Lk ? i + 1 : J->Lk) : J->Lk;
+    int64_t nsel = 0;
+    double next = -INFINITY;
+
+    if (J->eval_idx) {
+      /* index-evaluate: the kept set is given; recompute its scores. */
+      for (int64_t t = 0; t < K; ++t) {
+        int32_t j = J->eval_idx[r * K + t];
+        if (j < 0) continue;
+        if (j >= J->Lk) {
+          J->status = -3;
+          continue;
+        }
+        sel[nsel].j = j;
+        sel[nsel].s = dot_row(J, bh * J->Lk + j, qbuf);
+        nsel++;
+      }
+    } else if (J->vanilla) {
+      /* Eq. 1 / Eq. 2: every valid key is kept. */
+      for (int64_t j = 0; j < nvalid; ++j) {
+        sel[nsel].j = (int32_t)j;
+        sel[nsel].s = dot_row(J, bh * J->Lk + j, qbuf);
+        nsel++;
+      }
+    } else {
+      /* Eq. 4: bounded heap of the K+1 highest-ranked entries. */
+      int64_t cap = K + 1, n = 0;
+      for (int64_t j = 0; j < nvalid; ++j) {
+        entry e;
+        e.j = (int32_t)j;
+        e.s = dot_row(J, bh * J->Lk + j, qbuf);
+        if (n < cap) {
+          heap[n] = e;
+          heap_sift_up(heap, (int)n);
+          n++;
+        } else if (ranks_below(heap[0], e)) {
+          heap[0] = e;
+          heap_sift_down(heap, (int)n, 0);
+        }
+      }
+      memcpy(sel, heap, sizeof(entry) * (size_t)n);
+      qsort(sel, (size_t)n, sizeof(entry), cmp_rank_desc);
+      nsel = n > K ? K : n;
+      if (n > K) next = sel[K].s;
+    }
+    if (J->eval_idx || J->vanilla) qsort(sel, (size_t)nsel, sizeof(entry), cmp_rank_desc);
+
+    /* activation over the kept entries only (Eq. 4 / Eq. 3) */
+    if (J->act == ACT_SOFTMAX) {
+      double m = -INFINITY, z = 0.0;
+      for (int64_t t = 0; t < nsel; ++t)
+        if (sel[t].s > m) m = sel[t].s;
+      for (int64_t t = 0; t < nsel; ++t) {
+        w[t] = exp(sel[t].s - m);
+        z += w[t];
+      }
+      for (int64_t t = 0; t < nsel; ++t) w[t] /= z;
+    } else {
+      for (int64_t t = 0; t < nsel; ++t) w[t] = sel[t].s > 0.0 ? sel[t].s : 0.0;
+    }
+
+    /* weighted sum of the kept value rows */
+    double* o = J->out ? J->out + r * d : NULL;
+    if (o) {
+      for (int64_t c = 0; c < d; ++c) o[c] = 0.0;
+      for (int64_t t = 0; t < nsel; ++t) {
+        const int64_t vrow = bh * J->Lk + sel[t].j;
+        for (int64_t c = 0; c < d; ++c) o[c] += w[t] * widen(J->v, (size_t)(vrow * d + c), J->dtype);
+      }
+    }
+    if (J->idx && !J->vanilla) {
+      for (int64_t t = 0; t < K; ++t) J->idx[r * K + t] = t < nsel ? sel[t].j : -1;
+    }
+    if (J->score && !J->vanilla) {
+      for (int64_t t = 0; t < K; ++t) J->score[r * K + t] = t < nsel ? sel[t].s : -INFINITY;
+    }
+    if (J->next_score) J->next_score[r] = next;
+  }
+done:
+  free(qbuf);
+  free(heap);
+  free(sel);
+  free(w);
+  return NULL;
+}
+
+static int run(job proto, int nthreads) {
+  if (proto.d <= 0 || proto.Lq <= 0 || proto.Lk <= 0 || proto.topk < 1) return -2;
+  if (nthreads <= 0) nthreads = (int)sysconf(_SC_NPROCESSORS_ONLN);
+  if (nthreads < 1) nthreads = 1;
+  if (nthreads > proto.nrows) nthreads = (int)(proto.nrows > 0 ? proto.nrows : 1);
+  job* jobs = (job*)calloc((size_t)nthreads, sizeof(job));
+  pthread_t* th = (pthread_t*)calloc((size_t)nthreads, sizeof(pthread_t));
+  if (!jobs || !th) {
+    free(jobs);
+    free(th);
+    return -1;
+  }
+  int64_t per = (proto.nrows + nthreads - 1) / nthreads;
+  for (int t = 0; t < nthreads; ++t) {
+    jobs[t] = proto;
+    jobs[t].begin = (int64_t)t * per;
+    jobs[t].end = jobs[t].begin + per < proto.nrows ? jobs[t].begin + per : proto.nrows;
+    if (jobs[t].begin > jobs[t].end) jobs[t].begin = jobs[t].end;
+    jobs[t].status = 0;
+    pthread_create(&th[t], NULL, run_rows, &jobs[t]);
+  }
+  int status = 0;
+  for (int t = 0; t < nthreads; ++t) {
+    pthread_join(th[t], NULL);
+    if (jobs[t].status) status = jobs[t].status;
+  }
+  free(jobs);
+  free(th);
+  return status;
+}
+
+/* Top-k attention (Eq. 4) or, with act = ACT_RELU and B = H = 1, the
+ * top-k feed-forward layer (Eq. 3).  Rows are flattened (b, h, i) indices
+ * into [B*H*Lq]; rows == NULL means all of them in order.
+ * Outputs per listed row: out [d], idx [topk] (-1 padded), score [topk]
+ * (-inf padded), next_score = the (k+1)-th score or -inf. */
+int oracle_topk(int act, int dtype, const void* q, const void* k, const void* v, int64_t B, int64_t H,
+                int64_t Lq, int64_t Lk, int64_t d, int64_t topk, int causal, const int64_t* rows,
+                int64_t nrows, double* out, int32_t* idx, double* score, double* next_score,
+                int nthreads) {
+  job J;
+  memset(&J, 0, sizeof J);
+  J.act = act;
+  J.dtype = dtype;
+  J.q = q;
+  J.k = k;
+  J.v = v;
+  J.H = H;
+  J.Lq = Lq;
+  J.Lk = Lk;
+  J.d = d;
+  J.topk = topk;
+  J.causal = causal;
+  J.rows = rows;
+  J.nrows = rows ? nrows : B * H * Lq;
+  J.out = out;
+  J.idx = idx;
+  J.score = score;
+  J.next_score = next_score;
+  if (causal && Lq != Lk) return -2;
+  return run(J, nthreads);
+}
+
+/* Plain attention over every valid key (Eq. 1, with the causal mask of
+ * Eq. 2 when causal != 0).  Same row convention as oracle_topk. */
+int oracle_vanilla(int act, int dtype, const void* q, const void* k, const void* v, int64_t B, int64_t H,
+                   int64_t Lq, int64_t Lk, int64_t d, int causal, const int64_t* rows, int64_t nrows,
+                   double* out, int nthreads) {
+  job J;
+  memset(&J, 0, sizeof J);
+  J.act = act;
+  J.dtype = dtype;
+  J.q = q;
+  J.k = k;
+  J.v = v;
+  J.H = H;
+  J.Lq = Lq;
+  J.Lk = Lk;
+  J.d = d;
+  J.topk = Lk;
+  J.causal = causal;
+  J.vanilla = 1;
+  J.rows = rows;
+  J.nrows = rows ? nrows : B * H * Lq;
+  J.out = out;
+  if (causal && Lq != Lk) return -2;
+  return run(J, nthreads);
+}
+
+/* Index-evaluate: the kept set of each listed row is given in idx
+ * ([nrows][topk], -1 = empty slot); scores are recomputed in double and
+ * the activation and weighted sum follow Eq. 4 / Eq. 3 from there. */
+int oracle_eval_indices(int act, int dtype, const void* q, const void* k, const void* v, int64_t B,
+                        int64_t H, int64_t Lq, int64_t Lk, int64_t d, int64_t topk,
+                        const int64_t* rows, int64_t nrows, const int32_t* idx, double* out,
+                        double* score, int nthreads) {
+  job J;
+  memset(&J, 0, sizeof J);
+  J.act = act;
+  J.dtype = dtype;
+  J.q = q;
+  J.k = k;
+  J.v = v;
+  J.H = H;
+  J.Lq = Lq;
+  J.Lk = Lk;
+  J.d = d;
+  J.topk = topk;
+  J.rows = rows;
+  J.nrows = rows ? nrows : B * H * Lq;
+  J.eval_idx = idx;
+  J.out = out;
+  J.score = score;
+  return run(J, nthreads);
+}
+
+int oracle_hardware_threads(void) { return (int)sysconf(_SC_NPROCESSORS_ONLN); }

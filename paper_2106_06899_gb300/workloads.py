@@ -1,0 +1,138 @@
+"""Seeded synthetic inputs shaped like the paper's workloads.
+
+This module holds no arithmetic of the method: it only draws random tensors
+(on the CPU, with ``torch.Generator``) in the shapes and distributions below.
+Both the CUDA path's tests/benchmark and the CPU oracle read the very same
+host tensors from here.
+
+The shapes follow the paper's benchmark settings (Sec. 3): BERT-base
+multi-head attention (12 heads of 64 dims, Sec. 3 "Multi-head attention
+layer"), sequences up to 65,536 tokens with query chunks of 2^10 (Sec. 2.2
+"Query chunking"), a causal decoder layer, and a feed-forward layer with
+d_ff = 65,536 keys as in T5/UnifiedQA (Sec. 2.1 "Feed-forward as attention",
+Sec. 4.3).  None of the paper's datasets or trained weights are used; these
+random tensors stand in for them.
+
+Distributions (the temperature lambda = sqrt(d) of Eq. 1 is folded into the
+data, per the footnote to Eq. 1, by scaling both Q and K by d^-1/4):
+
+* ``normal``  -- Q, K ~ N(0, 1) * d^-1/4, V ~ N(0, 1).
+* ``lowrank`` -- Q = (G_q + s Z_q A) d^-1/4, K = (G_k + s Z_k A) d^-1/4 with
+  G ~ N(0, 1) [L, d], Z ~ N(0, 1) [L, 8], A [8, d] with orthonormal rows drawn
+  once per head, s = 2; V ~ N(0, 1).  The shared rank-8 part gives every
+  score row a heavier upper tail than the isotropic case.
+* ``ffn``     -- x ~ N(0, 1) [N, d_model]; W1, W2 ~ N(0, 1/d_model) [d_ff, d_model].
+"""
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, field, replace
+
+import torch
+
+LOWRANK_RANK = 8
+LOWRANK_SCALE = 2.0
+
+
+@dataclass(frozen=True)
+class Workload:
+    name: str
+    kind: str  # "attn" or "ffn"
+    dtype: str  # "f32" or "bf16"
+    seed: int
+    topk: int
+    # attention
+    B: int = 1
+    H: int = 1
+    Lq: int = 0
+    Lk: int = 0
+    d: int = 0
+    chunk: int = 0
+    causal: bool = False
+    dist: str = "normal"
+    # feed-forward
+    N: int = 0
+    d_model: int = 0
+    d_ff: int = 0
+    note: str = field(default="", compare=False)
+
+    @property
+    def rows(self) -> int:
+        return self.B * self.H * self.Lq if self.kind == "attn" else self.N
+
+    @property
+    def tokens(self) -> int:
+        return self.B * self.Lq if self.kind == "attn" else self.N
+
+    def with_(self, **kw) -> "Workload":
+        return replace(self, **kw)
+
+
+WORKLOADS = {
+    "tiny_fp32": Workload("tiny_fp32", "attn", "f32", seed=0, topk=32, B=1, H=1, Lq=512, Lk=512, d=64,
+                          chunk=128, note="tiny fp32 top-k attention"),
+    "bert_base": Workload("bert_base", "attn", "bf16", seed=1, topk=64, B=8, H=12, Lq=512, Lk=512, d=64,
+                          chunk=512, note="encoder-style BERT-base shape"),
+    "bert_base_all_keys": Workload("bert_base_all_keys", "attn", "bf16", seed=1, topk=512, B=8, H=12, Lq=512,
+                                   Lk=512, d=64, chunk=512, note="topk = Lk: must equal plain attention"),
+    "long_65k": Workload("long_65k", "attn", "bf16", seed=2, topk=64, B=1, H=12, Lq=65536, Lk=65536, d=64,
+                         chunk=1024, dist="lowrank", note="long-sequence top-64 attention, L = 65536"),
+    "causal_16k": Workload("causal_16k", "attn", "bf16", seed=3, topk=128, B=2, H=16, Lq=16384, Lk=16384,
+                           d=128, chunk=2048, causal=True, note="causal decoder-style, d = 128"),
+    "ffn_65k": Workload("ffn_65k", "ffn", "bf16", seed=4, topk=512, N=4096, d_model=1024, d_ff=65536,
+                        dist="ffn", note="top-k feed-forward, T5-large-like d_ff = 65536"),
+}
+
+
+def _torch_dtype(dtype: str) -> torch.dtype:
+    return {"f32": torch.float32, "bf16": torch.bfloat16}[dtype]
+
+
+def attention_inputs(B, H, Lq, Lk, d, *, dtype="bf16", seed=0, dist="normal"):
+    """(q [B,H,Lq,d], k [B,H,Lk,d], v [B,H,Lk,d]) on the CPU in ``dtype``."""
+    g = torch.Generator().manual_seed(int(seed))
+    scale = d ** -0.25
+    if dist == "normal":
+        q = torch.randn(B, H, Lq, d, generator=g)
+        k = torch.randn(B, H, Lk, d, generator=g)
+    elif dist == "lowrank":
+        r = min(LOWRANK_RANK, d)
+        basis = torch.randn(H, d, r, generator=g, dtype=torch.float64)
+        A = torch.linalg.qr(basis).Q.transpose(1, 2).to(torch.float32)  # [H, r, d], orthonormal rows
+        q = torch.randn(B, H, Lq, d, generator=g)
+        q += LOWRANK_SCALE * torch.randn(B, H, Lq, r, generator=g) @ A[None]
+        k = torch.randn(B, H, Lk, d, generator=g)
+        k += LOWRANK_SCALE * torch.randn(B, H, Lk, r, generator=g) @ A[None]
+    else:
+        raise ValueError(f"unknown distribution {dist!r}")
+    v = torch.randn(B, H, Lk, d, generator=g)
+    td = _torch_dtype(dtype)
+    return (q * scale).to(td).contiguous(), (k * scale).to(td).contiguous(), v.to(td).contiguous()
+
+
+def ffn_inputs(N, d_model, d_ff, *, dtype="bf16", seed=0):
+    """(x [N,d_model], W1 [d_ff,d_model], W2 [d_ff,d_model]) on the CPU in ``dtype``."""
+    g = torch.Generator().manual_seed(int(seed))
+    td = _torch_dtype(dtype)
+    x = torch.randn(N, d_model, generator=g)
+    std = 1.0 / math.sqrt(d_model)
+    w1 = torch.randn(d_ff, d_model, generator=g) * std
+    w2 = torch.randn(d_ff, d_model, generator=g) * std
+    return x.to(td).contiguous(), w1.to(td).contiguous(), w2.to(td).contiguous()
+
+
+def make_inputs(w: Workload):
+    if w.kind == "attn":
+        return attention_inputs(w.B, w.H, w.Lq, w.Lk, w.d, dtype=w.dtype, seed=w.seed, dist=w.dist)
+    return ffn_inputs(w.N, w.d_model, w.d_ff, dtype=w.dtype, seed=w.seed)
+
+
+def sample_rows(total: int, n: int, seed: int = 0) -> torch.Tensor:
+    """n distinct row indices in [0, total), sorted, always including the first and last row."""
+    n = min(n, total)
+    g = torch.Generator().manual_seed(int(seed) + 12345)
+    pick = torch.randperm(total, generator=g)[:n]
+    pick[0] = 0
+    if n > 1:
+        pick[1] = total - 1
+    return torch.unique(pick).sort().values
