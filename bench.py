@@ -1,0 +1,348 @@
+#!/usr/bin/env python3
+"""Throughput of top-k attention (arXiv 2106.06899, Eq. 4) on GB300.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
+
+One step is one call of the whole fused path (score GEMM, top-k selection,
+softmax over the k kept scores, value gather) over the full workload, inputs
+resident in device memory.  Default workload: B=1, H=12, L=65536, d=64,
+k=64, chunk 1024 (the long-sequence configuration).  Rank 0 prints one JSON
+line.  With N > 1 (torchrun, one rank per GPU) every rank runs an
+independent replica of the workload: the path has no exchange step, so there
+is no collective on the data path ("replicas only", weak scaling).
+
+--impl reference times the CPU oracle (fp64, all host cores) on bounded
+samples of the same workload: the only other implementation there is.
+"""
+from __future__ import annotations
+
+import argparse
+import csv
+import io
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "top-k attn tokens/s and QK^T TFLOP/s (% of bf16 peak) at L=65536, k=64"
+L2_BYTES = 129 * 1024 * 1024
+
+
+def parse_args():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=10)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="long_65k")
+    p.add_argument("--L", type=int, default=0, help="override Lq = Lk (profiling on a small case)")
+    p.add_argument("--e2e-steps", type=int, default=3)
+    p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU work budget of the oracle baseline")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-clocks", action="store_true")
+    return p.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            m = json.load(f)
+        return {"hbm_gbs": m["hbm_gbs"], "bf16": m["bf16_tflops"], "bf16_sustained": m["bf16_tflops_sustained"],
+                "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16": 1900.0, "bf16_sustained": 1700.0, "source": "fallback"}
+
+
+def workload(args):
+    from paper_2106_06899_gb300 import workloads as W
+
+    w = W.WORKLOADS[args.workload]
+    if args.L:
+        w = w.with_(Lq=args.L, Lk=args.L) if w.kind == "attn" else w.with_(d_ff=args.L)
+    return w
+
+
+def work_flops(w) -> float:
+    """Algorithmic score-GEMM FLOPs of one call (every score is computed, Sec. 5)."""
+    if w.kind == "ffn":
+        return 2.0 * w.N * w.d_ff * w.d_model
+    if w.causal:  # only unmasked pairs j <= i
+        pairs = w.Lq * (w.Lq + 1) / 2
+        return 2.0 * w.B * w.H * pairs * w.d
+    return 2.0 * w.B * w.H * w.Lq * w.Lk * w.d
+
+
+def config_dict(w, l2_note):
+    if w.kind == "ffn":
+        c = {"workload": w.name, "N": w.N, "d_model": w.d_model, "d_ff": w.d_ff, "topk": w.topk}
+    else:
+        c = {"workload": w.name, "B": w.B, "H": w.H, "Lq": w.Lq, "Lk": w.Lk, "d": w.d, "topk": w.topk,
+             "chunk": w.chunk, "causal": w.causal, "dist": w.dist}
+    c["l2"] = l2_note
+    c["parallelism"] = "replicas"
+    return c
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid: str | None):
+        self.uuid = uuid
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                                         text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        rows = []
+        for r in csv.reader(io.StringIO(out)):
+            r = [x.strip() for x in r]
+            if len(r) < 10:
+                continue
+            if self.uuid and self.uuid not in r[1]:
+                continue
+            rows.append(r)
+        if not rows:
+            return None
+        sm = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        mx = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[6 + i].lower() == "active"})
+        load = [s for s in sm if mx and s > 0.3 * max(mx)] or sm
+        return {"sm_mhz": statistics.median(load) if load else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
+
+
+# ------------------------------------------------------------------ oracle timing
+def oracle_rate(w, seconds: float, seed_rows: int = 0):
+    """Oracle tokens/s on a bounded sample of rows of the workload (same inputs, all host cores)."""
+    import oracle
+    from paper_2106_06899_gb300 import workloads as W
+
+    inputs = W.make_inputs(w)
+    cores = oracle.hardware_threads()
+
+    def run(nrows):
+        rows = W.sample_rows(w.rows, nrows, seed=seed_rows).numpy()
+        t0 = time.perf_counter()
+        if w.kind == "ffn":
+            oracle.ffn(*inputs, w.topk, rows=rows)
+        else:
+            oracle.topk_attention(*inputs, w.topk, causal=w.causal, rows=rows)
+        return len(rows), time.perf_counter() - t0
+
+    n, t = run(max(cores, 16))
+    target = max(int(n * seconds / max(t, 1e-3)), cores)
+    n, t = run(min(target, w.rows))
+    per_token = w.H if w.kind == "attn" else 1
+    return {"value": (n / per_token) / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n} of {w.rows} query rows (seeded sample), fp64 oracle, {t:.1f} s"}
+
+
+# ------------------------------------------------------------------ reference arm
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = workload(args)
+    import oracle
+    from paper_2106_06899_gb300 import workloads as W
+
+    inputs = W.make_inputs(w)
+    cores = oracle.hardware_threads()
+    per_token = w.H if w.kind == "attn" else 1
+
+    def step(nrows, seed):
+        rows = W.sample_rows(w.rows, nrows, seed=seed).numpy()
+        t0 = time.perf_counter()
+        if w.kind == "ffn":
+            oracle.ffn(*inputs, w.topk, rows=rows)
+        else:
+            oracle.topk_attention(*inputs, w.topk, causal=w.causal, rows=rows)
+        return len(rows), time.perf_counter() - t0
+
+    n, t = step(max(cores, 16), 0)
+    nrows = max(min(int(n * 2.0 / max(t, 1e-3)), w.rows), cores)  # about 2 s per step
+    for i in range(args.warmup):
+        step(nrows, 100 + i)
+    times = []
+    for i in range(args.steps):
+        n, t = step(nrows, 1000 + i)
+        times.append(t)
+    tt = sum(times)
+    value = (nrows * args.steps / per_token) / tt
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1000 * tt / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": config_dict(w, "host memory (CPU oracle)"),
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"{nrows} seeded query rows of {w.rows} per step"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------ our arm
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2106_06899_gb300 import topk as T
+    from paper_2106_06899_gb300 import workloads as W
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    def barrier():
+        if world > 1:
+            dist.barrier()
+
+    w = workload(args)
+    host = W.make_inputs(w.with_(seed=w.seed + rank))
+    dev = [t.cuda() for t in host]
+    in_bytes = sum(t.numel() * t.element_size() for t in host)
+    if w.kind == "ffn":
+        out = torch.empty(w.N, w.d_model, dtype=torch.float32, device="cuda")
+
+        def step():
+            T.topk_ffn_fwd(dev[0], dev[1], dev[2], out, w.topk)
+    else:
+        out = torch.empty_like(dev[0])
+
+        def step():
+            T.topk_attn_fwd(dev[0], dev[1], dev[2], out, w.topk, w.chunk, w.causal)
+
+    flush = None
+    if in_bytes <= 2 * L2_BYTES:
+        flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+        l2_note = "L2 flushed between steps (write of 2x L2 size), flush excluded by events"
+    else:
+        l2_note = f"inputs larger than L2 ({in_bytes / 2**20:.0f} MiB resident)"
+
+    for _ in range(args.warmup):
+        step()
+    T.topk_check()
+    launches_per_step = T.topk_last_launch_count()
+
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(local).uuid)
+    except Exception:
+        pass
+    sampler = ClockSampler(uuid)
+    if not args.no_clocks:
+        sampler.start()
+        time.sleep(0.3)
+    stream = torch.cuda.current_stream()
+    barrier()
+    torch.cuda.synchronize()
+    if flush is None:
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(args.steps):
+            step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = e0.elapsed_time(e1) / args.steps
+    else:
+        tot = 0.0
+        for _ in range(args.steps):
+            flush.fill_(1.0)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            step()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            tot += e0.elapsed_time(e1)
+        ms = tot / args.steps
+    barrier()
+    clocks = None if args.no_clocks else sampler.stop()
+    T.topk_check()
+
+    t_ms = torch.tensor([ms], device="cuda")
+    if world > 1:
+        dist.all_reduce(t_ms, op=dist.ReduceOp.MAX)
+    ms_max = float(t_ms.item())
+    value = world * w.tokens / (ms_max / 1e3)
+
+    # end to end through the host-buffer C-ABI entry: H2D copies, call, D2H copy, every step
+    pinned = [t.pin_memory() for t in host]
+    hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+    if w.kind == "ffn":
+        def e2e_step():
+            T.topk_ffn_fwd_host(pinned[0], pinned[1], pinned[2], hout, w.topk)
+    else:
+        def e2e_step():
+            T.topk_attn_fwd_host(pinned[0], pinned[1], pinned[2], hout, w.topk, w.chunk, w.causal)
+    e2e_step()
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        e2e_step()
+    e2e_s = (time.perf_counter() - t0) / args.e2e_steps
+    te = torch.tensor([e2e_s], device="cuda")
+    if world > 1:
+        dist.all_reduce(te, op=dist.ReduceOp.MAX)
+    e2e_value = world * w.tokens / float(te.item())
+
+    pk = peaks()
+    flops = work_flops(w)
+    achieved = flops / (ms_max / 1e3) / 1e12
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_max, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32", "data": "synthetic",
+        "config": config_dict(w, l2_note),
+        "tflops": achieved,
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": pk["bf16"], "unit": "TFLOP/s",
+                     "frac": achieved / pk["bf16"], "traffic": None,
+                     "peak_source": f"{pk['source']} bf16 dense (burst)",
+                     "kernel": "attn_tc_kernel" if w.kind == "attn" else "ffn kernels"},
+        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": in_bytes,
+                "d2h_bytes_per_step": out.numel() * out.element_size()},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clocks,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = oracle_rate(w, args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

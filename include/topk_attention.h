@@ -1,0 +1,156 @@
+/*
+ * topk_attention.h -- C ABI of libtopk.so: top-k attention and the top-k
+ * feed-forward layer (Gupta et al., "Memory-efficient Transformers via Top-k
+ * Attention", arXiv 2106.06899) on NVIDIA GB300 (sm_103a).
+ *
+ * Operations
+ *   topk_attn_fwd  -- Eq. 4 (Sec. 2.2):  out = softmax(top-k(Q K^T)) V, row by
+ *                     row, the softmax taken over the k kept entries only.
+ *                     The temperature of Eq. 1 is folded into Q by the caller
+ *                     (footnote to Eq. 1).  Optional causal mask, Eq. 2: key j
+ *                     is valid for query i iff j <= i.
+ *   topk_ffn_fwd   -- Eq. 3 with top-k (Sec. 2.1 "Feed-forward as attention"):
+ *                     out = sum over the k largest s_j = x . W1_j of
+ *                     ReLU(s_j) * W2_j.  Keys and values are the ROWS of W1
+ *                     and W2.
+ * Query chunking (Sec. 2.2 "Query chunking") bounds scheduling only: results
+ * never depend on `chunk`, and no [chunk x L_K] score matrix is ever stored
+ * in device memory.
+ *
+ * Selection rule: each row keeps the first k entries of the total order
+ * (score descending, key index ascending), i.e. ties go to the lower key
+ * index.  A causal row i with fewer than k valid keys keeps all i+1 of them.
+ *
+ * Conventions shared by every call
+ *   - Tensor pointers are DEVICE pointers (except the *_host entry points),
+ *     owned by the caller, contiguous, row-major, 16-byte aligned.
+ *   - Shapes: q, out [B, H, Lq, d]; k, v [B, H, Lk, d];
+ *             x [N, d_model]; W1, W2 [d_ff, d_model]; ffn out [N, d_model].
+ *   - dtype: TOPK_F32 (fp32 in/out, fp32 FMA scores, never TF32) or
+ *            TOPK_BF16 (bf16 in/out, fp32 accumulation).  The feed-forward
+ *            call takes bf16 inputs and writes fp32 output.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls
+ *     enqueue work and return without synchronising.
+ *   - Every argument is validated before anything is launched, so an error
+ *     return never leaves a partial write.
+ *   - Scratch, where a call needs it, is taken from the stream-ordered
+ *     allocator on `stream` and released on it; its size is reported by the
+ *     *_workspace_bytes queries and is linear in the number of query rows,
+ *     never proportional to Lq * Lk.
+ *
+ * Return codes: 0 on success, else one of the negative TOPK_ERR_* values;
+ * topk_error_string() describes them.
+ */
+#ifndef TOPK_ATTENTION_H
+#define TOPK_ATTENTION_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum { TOPK_F32 = 0, TOPK_BF16 = 1 } topk_dtype;
+
+enum {
+  TOPK_OK = 0,
+  TOPK_ERR_INVALID_ARG = -1, /* null pointer, non-positive size, topk < 1 or > keys, chunk < 1,
+                                causal with Lq != Lk, unknown dtype */
+  TOPK_ERR_UNSUPPORTED = -2, /* valid but not implemented: head size, topk above the
+                                kernel's limit, pointer not 16-byte aligned */
+  TOPK_ERR_CUDA = -3,        /* a CUDA runtime/driver call or a launch failed */
+  TOPK_ERR_TIMEOUT = -4,     /* a device pipeline wait ran out its time limit; the
+                                kernel stopped early and its outputs are invalid */
+  TOPK_ERR_WORKSPACE = -5,   /* a per-row candidate list ran out of room (needs
+                                more keys tied within one bf16 step of the k-th
+                                score than the list holds); outputs invalid */
+  TOPK_ERR_NO_DEVICE = -6    /* no usable sm_103 device */
+};
+
+/*
+ * Top-k attention forward, Eq. 4 (Sec. 2.2), optionally causal (Eq. 2).
+ *   q, k, v, out : device pointers, layouts above, element type `dtype`.
+ *   B, H         : batch and heads; every (b, h) is an independent problem.
+ *   Lq, Lk       : query and key counts (causal requires Lq == Lk).
+ *   d            : head size.  TOPK_BF16: 64 or 128.  TOPK_F32: 16, 32, 64, 128.
+ *   topk         : 1 <= topk <= Lk; the supported maximum is 512.
+ *   chunk        : query-chunk size (Sec. 2.2), >= 1; a scheduling hint only.
+ *   causal       : 0 or 1.
+ * Errors: TOPK_ERR_INVALID_ARG / TOPK_ERR_UNSUPPORTED before any launch;
+ *         TOPK_ERR_CUDA if a launch fails.  Device-side timeouts surface on
+ *         the next call or through topk_check().
+ */
+int topk_attn_fwd(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk,
+                  int d, int topk, int chunk, int causal, int dtype, void* stream);
+
+/*
+ * Same as topk_attn_fwd, and additionally writes, per query row, the kept
+ * key indices and their fp32 scores in selection order (score descending,
+ * index ascending).  idx [B, H, Lq, topk] int32, -1 padded; score same shape,
+ * fp32, -inf padded.  Either may be NULL.  Used for parity checks.
+ */
+int topk_attn_fwd_indices(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq,
+                          int Lk, int d, int topk, int chunk, int causal, int dtype, int32_t* idx,
+                          float* score, void* stream);
+
+/*
+ * Top-k feed-forward layer, Eq. 3 with the top-k of Eq. 4 and ReLU as the
+ * activation (Sec. 2.1, Sec. 2.2).
+ *   x  : [N, d_model] bf16 device pointer (the queries).
+ *   W1 : [d_ff, d_model] bf16; row j is key j.
+ *   W2 : [d_ff, d_model] bf16; row j is value j.
+ *   out: [N, d_model] fp32 device pointer.
+ *   d_model: a multiple of 64, at most 4096.  1 <= topk <= d_ff, topk <= 1024.
+ * Top-k is taken over the signed scores; ReLU is applied after selection.
+ */
+int topk_ffn_fwd(const void* x, const void* W1, const void* W2, void* out, int N, int d_model, int d_ff,
+                 int topk, void* stream);
+
+/* topk_ffn_fwd plus the kept indices [N, topk] int32 and scores [N, topk] fp32. */
+int topk_ffn_fwd_indices(const void* x, const void* W1, const void* W2, void* out, int N, int d_model,
+                         int d_ff, int topk, int32_t* idx, float* score, void* stream);
+
+/* Bytes of stream-ordered scratch the calls above take for these arguments
+ * (0 if none).  Returns 0 as well when the arguments are invalid. */
+size_t topk_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, int topk, int chunk, int dtype);
+size_t topk_ffn_workspace_bytes(int N, int d_model, int d_ff, int topk);
+
+/*
+ * End-to-end variants taking HOST pointers (pinned memory is fastest).  They
+ * stage the inputs into stream-ordered device memory, run the call above on
+ * `stream`, copy the result back and synchronise `stream` before returning.
+ * Sizes and dtypes as above.
+ */
+int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq,
+                       int Lk, int d, int topk, int chunk, int causal, int dtype, void* stream);
+int topk_ffn_fwd_host(const void* x, const void* W1, const void* W2, void* out, int N, int d_model,
+                      int d_ff, int topk, void* stream);
+
+/* Synchronises `stream` and returns the first device-side error recorded
+ * since the last check (TOPK_ERR_TIMEOUT / TOPK_ERR_WORKSPACE), clearing it;
+ * TOPK_ERR_CUDA if the stream itself reports an error; else TOPK_OK. */
+int topk_check(void* stream);
+
+/* Human-readable text for a return code (static storage). */
+const char* topk_error_string(int code);
+
+/* Number of kernel launches the last successful call on this host thread
+ * enqueued (for launch accounting in benchmarks). */
+int topk_last_launch_count(void);
+
+/* Testing hook: sets the device-side wait limit in microseconds for later
+ * calls (0 restores the default of 2 s) and returns the previous value. */
+long long topk_set_wait_limit_us(long long us);
+
+/* Testing hook: when `on` is non-zero, later tcgen05 attention launches
+ * withhold their second key tile, so that the consumers' bounded waits run
+ * out and the call reports TOPK_ERR_TIMEOUT through topk_check() without
+ * hanging the device.  Returns the previous setting. */
+int topk_debug_skip_arrive(int on);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TOPK_ATTENTION_H */

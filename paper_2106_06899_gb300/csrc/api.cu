@@ -1,0 +1,310 @@
+// api.cu -- the C ABI of libtopk.so (declared in include/topk_attention.h).
+//
+// Validates every argument before anything is enqueued, picks a kernel for
+// the shape, and launches it on the caller's stream.  Device pointers are
+// the caller's; the only state kept here is per-device: the device error
+// word (OR-ed by kernels whose bounded waits ran out) and the SM count.
+#include <atomic>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+
+#include "../../include/topk_attention.h"
+#include "kernels.h"
+
+namespace topk {
+
+namespace {
+
+__device__ unsigned g_device_error;  // one word per device, OR of kDevErr* flags
+
+constexpr int kMaxDevices = 64;
+struct DeviceState {
+  std::once_flag once;
+  unsigned* error_word = nullptr;
+  int num_sms = 0;
+  int cc_major = 0, cc_minor = 0;
+  bool ok = false;
+};
+DeviceState g_dev[kMaxDevices];
+
+std::atomic<long long> g_wait_limit_us{0};
+std::atomic<int> g_debug_skip_arrive{0};
+thread_local int t_last_launches = 0;
+
+DeviceState* device_state() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  DeviceState& s = g_dev[dev];
+  std::call_once(s.once, [&s, dev]() {
+    cudaDeviceProp p;
+    if (cudaGetDeviceProperties(&p, dev) != cudaSuccess) return;
+    s.num_sms = p.multiProcessorCount;
+    s.cc_major = p.major;
+    s.cc_minor = p.minor;
+    void* addr = nullptr;
+    if (cudaGetSymbolAddress(&addr, g_device_error) != cudaSuccess) return;
+    s.error_word = static_cast<unsigned*>(addr);
+    s.ok = true;
+  });
+  return s.ok ? &s : nullptr;
+}
+
+DevCtl make_ctl(DeviceState* s) {
+  DevCtl c;
+  c.error = s->error_word;
+  const long long us = g_wait_limit_us.load();
+  c.wait_limit_ns = static_cast<unsigned long long>(us > 0 ? us : 2000000LL) * 1000ull;
+  c.debug_skip_arrive = g_debug_skip_arrive.load();
+  return c;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+int validate_attn(const AttnArgs& a) {
+  if (!a.q || !a.k || !a.v || !a.out) return TOPK_ERR_INVALID_ARG;
+  if (a.B <= 0 || a.H <= 0 || a.Lq <= 0 || a.Lk <= 0 || a.d <= 0) return TOPK_ERR_INVALID_ARG;
+  if (a.topk < 1 || a.topk > a.Lk || a.chunk < 1) return TOPK_ERR_INVALID_ARG;
+  if (a.causal != 0 && a.causal != 1) return TOPK_ERR_INVALID_ARG;
+  if (a.causal && a.Lq != a.Lk) return TOPK_ERR_INVALID_ARG;
+  if (a.dtype != TOPK_F32 && a.dtype != TOPK_BF16) return TOPK_ERR_INVALID_ARG;
+  const long long BH = static_cast<long long>(a.B) * a.H;
+  if (BH > (1 << 30) || static_cast<long long>(a.Lq) * BH > (1ll << 40)) return TOPK_ERR_UNSUPPORTED;
+  if (a.topk > kSimtMaxK) return TOPK_ERR_UNSUPPORTED;
+  if (a.dtype == TOPK_BF16 && a.d != 64 && a.d != 128) return TOPK_ERR_UNSUPPORTED;
+  if (a.dtype == TOPK_F32 && a.d != 16 && a.d != 32 && a.d != 64 && a.d != 128) return TOPK_ERR_UNSUPPORTED;
+  if (!aligned16(a.q) || !aligned16(a.k) || !aligned16(a.v) || !aligned16(a.out)) return TOPK_ERR_UNSUPPORTED;
+  return TOPK_OK;
+}
+
+int run_attn(const AttnArgs& a, cudaStream_t st) {
+  int rc = validate_attn(a);
+  if (rc) return rc;
+  DeviceState* dev = device_state();
+  if (!dev) return TOPK_ERR_NO_DEVICE;
+  if (dev->cc_major != 10 || dev->cc_minor != 3) return TOPK_ERR_NO_DEVICE;
+  const DevCtl ctl = make_ctl(dev);
+  int n = attn_tc(a, ctl, dev->num_sms, st);
+  if (n == 0) n = attn_simt(a, st);
+  if (n == 0) return TOPK_ERR_UNSUPPORTED;
+  if (n < 0) return TOPK_ERR_CUDA;
+  t_last_launches = n;
+  return TOPK_OK;
+}
+
+int validate_ffn(const FfnArgs& a) {
+  if (!a.x || !a.W1 || !a.W2 || !a.out) return TOPK_ERR_INVALID_ARG;
+  if (a.N <= 0 || a.d_model <= 0 || a.d_ff <= 0) return TOPK_ERR_INVALID_ARG;
+  if (a.topk < 1 || a.topk > a.d_ff) return TOPK_ERR_INVALID_ARG;
+  if (a.d_model % 64 != 0 || a.d_model > 4096) return TOPK_ERR_UNSUPPORTED;
+  if (a.topk > 1024) return TOPK_ERR_UNSUPPORTED;
+  if (!aligned16(a.x) || !aligned16(a.W1) || !aligned16(a.W2) || !aligned16(a.out)) return TOPK_ERR_UNSUPPORTED;
+  return TOPK_OK;
+}
+
+int run_ffn(FfnArgs a, cudaStream_t st) {
+  int rc = validate_ffn(a);
+  if (rc) return rc;
+  DeviceState* dev = device_state();
+  if (!dev) return TOPK_ERR_NO_DEVICE;
+  if (dev->cc_major != 10 || dev->cc_minor != 3) return TOPK_ERR_NO_DEVICE;
+  const DevCtl ctl = make_ctl(dev);
+  const size_t ws = ffn_workspace_bytes(a.N, a.d_model, a.d_ff, a.topk);
+  void* buf = nullptr;
+  if (ws) {
+    if (cudaMallocAsync(&buf, ws, st) != cudaSuccess) return TOPK_ERR_CUDA;
+  }
+  a.workspace = buf;
+  a.workspace_bytes = ws;
+  int n = ffn_tc(a, ctl, dev->num_sms, st);
+  if (buf) cudaFreeAsync(buf, st);
+  if (n == 0) return TOPK_ERR_UNSUPPORTED;
+  if (n < 0) return TOPK_ERR_CUDA;
+  t_last_launches = n;
+  return TOPK_OK;
+}
+
+size_t elem_bytes(int dtype) { return dtype == TOPK_F32 ? 4 : 2; }
+
+}  // namespace
+
+EncodeTiledFn encode_tiled_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, []() {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
+                       uint32_t box1) {
+  EncodeTiledFn enc = encode_tiled_fn();
+  if (!enc) return false;
+  cuuint64_t dims[3] = {dim0, dim1, dim2};
+  cuuint64_t strides[2] = {dim0 * 2, dim0 * dim1 * 2};
+  cuuint32_t box[3] = {64, box1, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace topk
+
+using namespace topk;
+
+extern "C" {
+
+int topk_attn_fwd(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk, int d,
+                  int topk, int chunk, int causal, int dtype, void* stream) {
+  AttnArgs a{q, k, v, out, B, H, Lq, Lk, d, topk, chunk, causal, dtype, nullptr, nullptr};
+  return run_attn(a, static_cast<cudaStream_t>(stream));
+}
+
+int topk_attn_fwd_indices(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk,
+                          int d, int topk, int chunk, int causal, int dtype, int32_t* idx, float* score,
+                          void* stream) {
+  if ((idx && !aligned16(idx)) || (score && !aligned16(score))) return TOPK_ERR_UNSUPPORTED;
+  AttnArgs a{q, k, v, out, B, H, Lq, Lk, d, topk, chunk, causal, dtype, idx, score};
+  return run_attn(a, static_cast<cudaStream_t>(stream));
+}
+
+int topk_ffn_fwd(const void* x, const void* W1, const void* W2, void* out, int N, int d_model, int d_ff, int topk,
+                 void* stream) {
+  FfnArgs a{x, W1, W2, static_cast<float*>(out), N, d_model, d_ff, topk, nullptr, nullptr, nullptr, 0};
+  return run_ffn(a, static_cast<cudaStream_t>(stream));
+}
+
+int topk_ffn_fwd_indices(const void* x, const void* W1, const void* W2, void* out, int N, int d_model, int d_ff,
+                         int topk, int32_t* idx, float* score, void* stream) {
+  FfnArgs a{x, W1, W2, static_cast<float*>(out), N, d_model, d_ff, topk, idx, score, nullptr, 0};
+  return run_ffn(a, static_cast<cudaStream_t>(stream));
+}
+
+size_t topk_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, int topk, int chunk, int dtype) {
+  AttnArgs a{reinterpret_cast<void*>(16), reinterpret_cast<void*>(16), reinterpret_cast<void*>(16),
+             reinterpret_cast<void*>(16), B, H, Lq, Lk, d, topk, chunk, 0, dtype, nullptr, nullptr};
+  (void)validate_attn(a);
+  return 0;  // the attention kernels keep their state in shared memory and TMEM
+}
+
+size_t topk_ffn_workspace_bytes(int N, int d_model, int d_ff, int topk) {
+  FfnArgs a{reinterpret_cast<void*>(16), reinterpret_cast<void*>(16), reinterpret_cast<void*>(16),
+            reinterpret_cast<float*>(16), N, d_model, d_ff, topk, nullptr, nullptr, nullptr, 0};
+  if (validate_ffn(a) != TOPK_OK) return 0;
+  return ffn_workspace_bytes(N, d_model, d_ff, topk);
+}
+
+int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk, int d,
+                       int topk, int chunk, int causal, int dtype, void* stream) {
+  if (!q || !k || !v || !out) return TOPK_ERR_INVALID_ARG;
+  if (B <= 0 || H <= 0 || Lq <= 0 || Lk <= 0 || d <= 0) return TOPK_ERR_INVALID_ARG;
+  AttnArgs chk{reinterpret_cast<void*>(16), reinterpret_cast<void*>(16), reinterpret_cast<void*>(16),
+               reinterpret_cast<void*>(16), B, H, Lq, Lk, d, topk, chunk, causal, dtype, nullptr, nullptr};
+  int rc = validate_attn(chk);
+  if (rc) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t eb = elem_bytes(dtype);
+  const size_t qb = static_cast<size_t>(B) * H * Lq * d * eb, kb = static_cast<size_t>(B) * H * Lk * d * eb;
+  void *dq = nullptr, *dk = nullptr, *dv = nullptr, *dout = nullptr;
+  if (cudaMallocAsync(&dq, qb, st) != cudaSuccess || cudaMallocAsync(&dk, kb, st) != cudaSuccess ||
+      cudaMallocAsync(&dv, kb, st) != cudaSuccess || cudaMallocAsync(&dout, qb, st) != cudaSuccess) {
+    rc = TOPK_ERR_CUDA;
+  } else if (cudaMemcpyAsync(dq, q, qb, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+             cudaMemcpyAsync(dk, k, kb, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+             cudaMemcpyAsync(dv, v, kb, cudaMemcpyHostToDevice, st) != cudaSuccess) {
+    rc = TOPK_ERR_CUDA;
+  } else {
+    rc = topk_attn_fwd(dq, dk, dv, dout, B, H, Lq, Lk, d, topk, chunk, causal, dtype, stream);
+    if (rc == TOPK_OK && cudaMemcpyAsync(out, dout, qb, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+      rc = TOPK_ERR_CUDA;
+  }
+  const int launches = t_last_launches;
+  if (dq) cudaFreeAsync(dq, st);
+  if (dk) cudaFreeAsync(dk, st);
+  if (dv) cudaFreeAsync(dv, st);
+  if (dout) cudaFreeAsync(dout, st);
+  if (cudaStreamSynchronize(st) != cudaSuccess && rc == TOPK_OK) rc = TOPK_ERR_CUDA;
+  t_last_launches = launches;
+  return rc;
+}
+
+int topk_ffn_fwd_host(const void* x, const void* W1, const void* W2, void* out, int N, int d_model, int d_ff,
+                      int topk, void* stream) {
+  if (!x || !W1 || !W2 || !out) return TOPK_ERR_INVALID_ARG;
+  FfnArgs chk{reinterpret_cast<void*>(16), reinterpret_cast<void*>(16), reinterpret_cast<void*>(16),
+              reinterpret_cast<float*>(16), N, d_model, d_ff, topk, nullptr, nullptr, nullptr, 0};
+  int rc = validate_ffn(chk);
+  if (rc) return rc;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const size_t xb = static_cast<size_t>(N) * d_model * 2, wb = static_cast<size_t>(d_ff) * d_model * 2;
+  const size_t ob = static_cast<size_t>(N) * d_model * 4;
+  void *dx = nullptr, *d1 = nullptr, *d2 = nullptr, *dout = nullptr;
+  if (cudaMallocAsync(&dx, xb, st) != cudaSuccess || cudaMallocAsync(&d1, wb, st) != cudaSuccess ||
+      cudaMallocAsync(&d2, wb, st) != cudaSuccess || cudaMallocAsync(&dout, ob, st) != cudaSuccess) {
+    rc = TOPK_ERR_CUDA;
+  } else if (cudaMemcpyAsync(dx, x, xb, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+             cudaMemcpyAsync(d1, W1, wb, cudaMemcpyHostToDevice, st) != cudaSuccess ||
+             cudaMemcpyAsync(d2, W2, wb, cudaMemcpyHostToDevice, st) != cudaSuccess) {
+    rc = TOPK_ERR_CUDA;
+  } else {
+    rc = topk_ffn_fwd(dx, d1, d2, dout, N, d_model, d_ff, topk, stream);
+    if (rc == TOPK_OK && cudaMemcpyAsync(out, dout, ob, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+      rc = TOPK_ERR_CUDA;
+  }
+  const int launches = t_last_launches;
+  if (dx) cudaFreeAsync(dx, st);
+  if (d1) cudaFreeAsync(d1, st);
+  if (d2) cudaFreeAsync(d2, st);
+  if (dout) cudaFreeAsync(dout, st);
+  if (cudaStreamSynchronize(st) != cudaSuccess && rc == TOPK_OK) rc = TOPK_ERR_CUDA;
+  t_last_launches = launches;
+  return rc;
+}
+
+int topk_check(void* stream) {
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(st) != cudaSuccess) return TOPK_ERR_CUDA;
+  DeviceState* dev = device_state();
+  if (!dev) return TOPK_ERR_NO_DEVICE;
+  unsigned word = 0;
+  if (cudaMemcpy(&word, dev->error_word, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess) return TOPK_ERR_CUDA;
+  if (word) {
+    const unsigned zero = 0;
+    if (cudaMemcpy(dev->error_word, &zero, sizeof zero, cudaMemcpyHostToDevice) != cudaSuccess)
+      return TOPK_ERR_CUDA;
+  }
+  if (word & kDevErrTimeout) return TOPK_ERR_TIMEOUT;
+  if (word & kDevErrWorkspace) return TOPK_ERR_WORKSPACE;
+  return TOPK_OK;
+}
+
+const char* topk_error_string(int code) {
+  switch (code) {
+    case TOPK_OK: return "success";
+    case TOPK_ERR_INVALID_ARG: return "invalid argument";
+    case TOPK_ERR_UNSUPPORTED: return "unsupported shape, dtype, topk or alignment";
+    case TOPK_ERR_CUDA: return "CUDA error";
+    case TOPK_ERR_TIMEOUT: return "device pipeline wait timed out; outputs invalid";
+    case TOPK_ERR_WORKSPACE: return "per-row candidate list overflowed; outputs invalid";
+    case TOPK_ERR_NO_DEVICE: return "no usable sm_103 device";
+    default: return "unknown error code";
+  }
+}
+
+int topk_last_launch_count(void) { return t_last_launches; }
+
+long long topk_set_wait_limit_us(long long us) { return g_wait_limit_us.exchange(us < 0 ? 0 : us); }
+
+// Testing hook (not in the public header): makes the tcgen05 attention
+// producer withhold its second key tile so that the consumers' bounded waits
+// run out; returns the previous setting.
+int topk_debug_skip_arrive(int on) { return g_debug_skip_arrive.exchange(on ? 1 : 0); }
+
+}  // extern "C"

@@ -1,0 +1,348 @@
+// attn_tc.cu -- fused top-k attention (Eq. 4) for bf16 inputs on sm_103a.
+//
+// One persistent CTA per SM walks work units (b, h, 128-query tile).  For a
+// unit the query tile Q_C (Sec. 2.2 "Query chunking", C = 128) is loaded once
+// by TMA, then the keys stream through in tiles of N:
+//
+//   warp 0      TMA producer: Q tile, then K tiles into a shared-memory ring
+//   warp 1      MMA issuer: S = Q_C K_tile^T with tcgen05.mma (bf16 in, fp32
+//               accumulate) into one of two TMEM accumulators [128 x N]
+//   warps 2..5  selection: thread t of warp w owns TMEM lane / query row
+//               32*(w%4)+t; it reads its N scores with tcgen05.ld and offers
+//               them to its row's top-k heap (select.cuh); after the last
+//               key tile it sorts the k kept keys, applies the softmax over
+//               them and gathers the matching value rows (fp32 accumulate).
+//
+// The score tile never leaves TMEM/registers: no [C x Lk] matrix is written
+// to device memory (Sec. 2.2 "Query chunking": memory O(C Lk) becomes
+// O(C k) here, in shared memory).  The scale of Eq. 1 is folded into Q by
+// the caller.  Causal masking (Eq. 2) skips key tiles past the query tile
+// and masks keys j > i inside the diagonal tile.
+//
+// Every pipeline wait is bounded (common.cuh); on expiry the CTA stops,
+// drains its in-flight copies and MMAs, frees TMEM and returns.
+#include "kernels.h"
+#include "select.cuh"
+
+namespace topk {
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int kThreads = 192;
+
+template <int D>
+struct TcShape;
+template <>
+struct TcShape<64> {
+  static constexpr int N = 256;
+  static constexpr int S = 2;
+};
+template <>
+struct TcShape<128> {
+  static constexpr int N = 128;
+  static constexpr int S = 2;
+};
+
+template <int D>
+struct Layout {
+  static constexpr int N = TcShape<D>::N;
+  static constexpr int S = TcShape<D>::S;
+  static constexpr int R = D / 64;  // 128-byte column blocks per row
+  static constexpr uint32_t Q_BYTES = BM * D * 2;
+  static constexpr uint32_t KST_BYTES = N * D * 2;
+  static constexpr size_t OFF_Q = 0;
+  static constexpr size_t OFF_K = OFF_Q + Q_BYTES;
+  static constexpr size_t OFF_HEAP = OFF_K + static_cast<size_t>(S) * KST_BYTES;
+  static constexpr int NBARS = 2 * S + 7;
+  static constexpr size_t CTRL_BYTES = 256;
+  static size_t bytes(int topk) { return 1024 + OFF_HEAP + static_cast<size_t>(topk) * BM * 8 + CTRL_BYTES; }
+};
+
+// Waits on an mbarrier phase with lane 0 of the warp and broadcasts the
+// outcome, so that the whole warp leaves together.
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, const DevCtl& ctl,
+                                          volatile int* abort_flag) {
+  int ok = 0;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, ctl, abort_flag) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  return ok != 0;
+}
+
+// Bounded wait that ignores the abort flag: used only to drain in-flight
+// asynchronous work before the CTA exits.
+__device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, const DevCtl& ctl) {
+  const unsigned long long t0 = global_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_ns() - t0 > ctl.wait_limit_ns) {
+      atomicOr(ctl.error, kDevErrTimeout);
+      return;
+    }
+  }
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_tc_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmk,
+                   const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ out, int BH, int Lq, int Lk,
+                   int topk, int causal, int n_units, int32_t* __restrict__ idx, float* __restrict__ score,
+                   DevCtl ctl) {
+  using L = Layout<D>;
+  constexpr int N = L::N, S = L::S, R = L::R;
+  constexpr uint32_t IDESC = idesc_bf16_f32(BM, N);
+  constexpr uint32_t TMEM_COLS = 2 * N;
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint8_t* q_s = smem + L::OFF_Q;
+  uint8_t* k_s = smem + L::OFF_K;
+  uint64_t* heap_mem = reinterpret_cast<uint64_t*>(smem + L::OFF_HEAP);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::OFF_HEAP + static_cast<size_t>(topk) * BM * 8);
+  uint64_t* full_k = bars;
+  uint64_t* empty_k = bars + S;
+  uint64_t* q_full = bars + 2 * S;
+  uint64_t* q_empty = bars + 2 * S + 1;
+  uint64_t* acc_full = bars + 2 * S + 2;   // [2]
+  uint64_t* acc_empty = bars + 2 * S + 4;  // [2]
+  uint64_t* drain = bars + 2 * S + 6;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + L::NBARS);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < S; ++s) {
+      mbar_init(&full_k[s], 1);
+      mbar_init(&empty_k[s], 1);
+    }
+    mbar_init(q_full, 1);
+    mbar_init(q_empty, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&acc_full[b], 1);
+      mbar_init(&acc_empty[b], 4);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) tmem_alloc(tmem_slot, TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  const int n_qt = (Lq + BM - 1) / BM;
+  auto decode = [&](int u, int& bh, int& qt) {
+    if (causal) {  // heaviest query tiles first
+      qt = n_qt - 1 - u / BH;
+      bh = u % BH;
+    } else {  // consecutive units share a head, so its K/V stay in L2
+      bh = u / n_qt;
+      qt = u % n_qt;
+    }
+  };
+  auto key_tiles = [&](int qt) {
+    const int kend = causal ? min(Lk, (qt + 1) * BM) : Lk;
+    return (kend + N - 1) / N;
+  };
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      tma_prefetch_desc(&tmq);
+      tma_prefetch_desc(&tmk);
+    }
+    uint32_t it = 0, q_issued = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+      int bh, qt;
+      decode(u, bh, qt);
+      if (!warp_wait(q_empty, (q_issued & 1u) ^ 1u, ctl, abort_flag)) {
+        ok = false;
+        break;
+      }
+      if (lane == 0) {
+        mbar_arrive_expect_tx(q_full, L::Q_BYTES);
+        for (int r = 0; r < R; ++r) tma_load_3d(q_s + r * BM * 128, &tmq, q_full, r * 64, qt * BM, bh);
+      }
+      ++q_issued;
+      const int nk = key_tiles(qt);
+      for (int kt = 0; kt < nk; ++kt) {
+        const int s = it % S;
+        const uint32_t ph = (it / S) & 1u;
+        if (!warp_wait(&empty_k[s], ph ^ 1u, ctl, abort_flag)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) {
+          if (ctl.debug_skip_arrive && it == 1) {
+            // testing hook: withhold this stage so the consumers' waits run out
+          } else {
+            mbar_arrive_expect_tx(&full_k[s], L::KST_BYTES);
+            for (int r = 0; r < R; ++r)
+              tma_load_3d(k_s + static_cast<size_t>(s) * L::KST_BYTES + r * N * 128, &tmk, &full_k[s], r * 64,
+                          kt * N, bh);
+          }
+        }
+        ++it;
+      }
+    }
+    // drain: every issued copy must have landed before the CTA may exit
+    if (lane == 0) {
+      for (uint32_t back = 1; back <= static_cast<uint32_t>(S) && back <= it; ++back) {
+        const uint32_t t = it - back;
+        if (ctl.debug_skip_arrive && t == 1) continue;
+        mbar_drain(&full_k[t % S], (t / S) & 1u, ctl);
+      }
+      if (q_issued > 0) mbar_drain(q_full, (q_issued - 1) & 1u, ctl);
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    uint32_t it = 0, acc_it = 0, qi = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x, ++qi) {
+      int bh, qt;
+      decode(u, bh, qt);
+      if (!warp_wait(q_full, qi & 1u, ctl, abort_flag)) {
+        ok = false;
+        break;
+      }
+      tc_fence_after();
+      const int nk = key_tiles(qt);
+      for (int kt = 0; kt < nk; ++kt, ++it, ++acc_it) {
+        const int s = it % S;
+        if (!warp_wait(&full_k[s], (it / S) & 1u, ctl, abort_flag)) {
+          ok = false;
+          break;
+        }
+        const int b = acc_it & 1;
+        if (!warp_wait(&acc_empty[b], ((acc_it >> 1) & 1u) ^ 1u, ctl, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        if (lane == 0) {
+          const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(b * N);
+          const uint32_t qa = smem_u32(q_s);
+          const uint32_t ka = smem_u32(k_s + static_cast<size_t>(s) * L::KST_BYTES);
+#pragma unroll
+          for (int st = 0; st < D / 16; ++st) {
+            const uint32_t r = st / 4, off = (st % 4) * 32;
+            mma_bf16_ss(d_tmem, sdesc_k128(qa + r * BM * 128 + off), sdesc_k128(ka + r * N * 128 + off), IDESC,
+                        st > 0 ? 1u : 0u);
+          }
+          mma_commit(&empty_k[s]);
+          mma_commit(&acc_full[b]);
+        }
+        __syncwarp();
+      }
+      if (!ok) break;
+      if (lane == 0) mma_commit(q_empty);
+      __syncwarp();
+    }
+    // drain: all issued MMAs must complete before TMEM is freed
+    if (lane == 0) {
+      mma_commit(drain);
+      mbar_drain(drain, 0, ctl);
+    }
+    __syncwarp();
+  } else {
+    // ------------------------------------------------------------ selection
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
+    uint32_t acc_it = 0;
+    RowHeap<BM> heap;
+    bool ok = true;
+    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+      int bh, qt;
+      decode(u, bh, qt);
+      const int i_row = qt * BM + row;
+      heap.init(heap_mem, row, topk);
+      const int nk = key_tiles(qt);
+      const uint32_t lim = static_cast<uint32_t>(causal ? min(i_row + 1, Lk) : Lk);
+      const int lim_min = causal ? min(qt * BM + 1, Lk) : Lk;
+      for (int kt = 0; kt < nk; ++kt, ++acc_it) {
+        const int b = acc_it & 1;
+        if (!warp_wait(&acc_full[b], (acc_it >> 1) & 1u, ctl, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(b * N);
+        const uint32_t jt = static_cast<uint32_t>(kt * N);
+#pragma unroll 1
+        for (int c = 0; c < N / 32; ++c) {
+          float vals[32];
+          __syncwarp();
+          tmem_ld32(taddr + c * 32, vals);
+          tmem_wait_ld();
+          if (c == N / 32 - 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acc_empty[b]);
+          }
+          const uint32_t j0 = jt + static_cast<uint32_t>(c * 32);
+          if (static_cast<int>(j0) + 32 > lim_min) mask32(vals, j0, lim);
+          heap.offer32(vals, j0);
+        }
+      }
+      if (!ok) break;
+      if (i_row < Lq) {
+        heap.sort_desc();
+        const size_t orow = static_cast<size_t>(bh) * Lq + i_row;
+        softmax_gather_store<__nv_bfloat16, D, BM>(heap, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
+        if (idx || score)
+          write_selection(heap, idx ? idx + orow * topk : nullptr, score ? score + orow * topk : nullptr);
+      }
+      __syncwarp();
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, TMEM_COLS);
+  }
+}
+
+template <int D>
+int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
+  using L = Layout<D>;
+  const int BH = a.B * a.H;
+  CUtensorMap tmq, tmk;
+  if (!make_tmap_bf16_3d(&tmq, a.q, D, a.Lq, BH, BM)) return -1;
+  if (!make_tmap_bf16_3d(&tmk, a.k, D, a.Lk, BH, L::N)) return -1;
+  const int n_units = BH * ((a.Lq + BM - 1) / BM);
+  // At least 120 KB so that a second CTA never shares the SM: each CTA takes
+  // all TMEM columns it needs for its whole (persistent) lifetime.
+  const size_t smem = L::bytes(a.topk) > 120 * 1024 ? L::bytes(a.topk) : 120 * 1024;
+  auto kern = attn_tc_kernel<D>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
+      cudaSuccess)
+    return -1;
+  const int grid = n_units < num_sms ? n_units : num_sms;
+  kern<<<grid, kThreads, smem, st>>>(tmq, tmk, static_cast<const __nv_bfloat16*>(a.v),
+                                     static_cast<__nv_bfloat16*>(a.out), BH, a.Lq, a.Lk, a.topk, a.causal, n_units,
+                                     a.idx, a.score, ctl);
+  return cudaGetLastError() == cudaSuccess ? 1 : -1;
+}
+
+}  // namespace
+
+bool attn_tc_supports(const AttnArgs& a) {
+  if (a.dtype != 1 || a.topk > kTcMaxK) return false;
+  if (a.d == 64) return Layout<64>::bytes(a.topk) <= 232448;
+  if (a.d == 128) return Layout<128>::bytes(a.topk) <= 232448;
+  return false;
+}
+
+int attn_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
+  if (!attn_tc_supports(a)) return 0;
+  return a.d == 64 ? launch_tc<64>(a, ctl, num_sms, st) : launch_tc<128>(a, ctl, num_sms, st);
+}
+
+}  // namespace topk

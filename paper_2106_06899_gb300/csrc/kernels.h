@@ -1,0 +1,62 @@
+// kernels.h -- internal interface between the C-ABI layer (api.cu) and the
+// kernel translation units.  Not part of the public ABI.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "common.cuh"
+
+namespace topk {
+
+// topk above this uses 32-row CTAs on the SIMT path (heap memory is
+// topk x rows x 8 bytes of shared memory).
+constexpr int kSimtSmallRowsMaxK = 128;
+constexpr int kSimtMaxK = 512;
+// tcgen05 attention path limit (heap for 128 rows in shared memory)
+constexpr int kTcMaxK = 128;
+
+struct AttnArgs {
+  const void* q;
+  const void* k;
+  const void* v;
+  void* out;
+  int B, H, Lq, Lk, d, topk, chunk, causal, dtype;
+  int32_t* idx;
+  float* score;
+};
+
+struct FfnArgs {
+  const void* x;
+  const void* W1;
+  const void* W2;
+  float* out;
+  int N, d_model, d_ff, topk;
+  int32_t* idx;
+  float* score;
+  void* workspace;
+  size_t workspace_bytes;
+};
+
+// Each launcher returns the number of kernel launches (> 0) on success,
+// 0 if it does not serve the given shape, -1 on a CUDA error.
+int attn_simt(const AttnArgs& a, cudaStream_t st);
+int attn_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st);
+bool attn_tc_supports(const AttnArgs& a);
+
+size_t ffn_workspace_bytes(int N, int d_model, int d_ff, int topk);
+int ffn_tc(const FfnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st);
+
+// Driver entry point for cuTensorMapEncodeTiled (resolved once, no libcuda link).
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_tiled_fn();
+
+// 3-D bf16 tensor map [dim2][dim1][dim0] (dim0 innermost, contiguous) with a
+// box of {64, box1, 1} and 128-byte swizzle.  Returns false on failure.
+bool make_tmap_bf16_3d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint64_t dim2,
+                       uint32_t box1);
+
+}  // namespace topk

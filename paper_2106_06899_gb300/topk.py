@@ -1,0 +1,213 @@
+"""Thin ctypes binding of libtopk.so (include/topk_attention.h).
+
+Argument marshalling only: every step of the computation runs in the CUDA
+library.  Functions carry the C-ABI names; they take torch tensors, read
+sizes from their shapes, pass raw pointers and raise ``TopkError`` on a
+non-zero return code.  There is no fallback: if libtopk.so is missing or
+no GB300 is present the calls fail loudly.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libtopk.so")
+
+TOPK_F32, TOPK_BF16 = 0, 1
+_lock = threading.Lock()
+_lib = None
+
+
+class TopkError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = code
+        super().__init__(f"{where}: {error_string(code)} (code {code})")
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded libtopk.so.  Raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise ImportError(f"{LIB_PATH} is not built; run `python -m paper_2106_06899_gb300.build` "
+                                  "(nvcc for sm_103a) first")
+            L = ctypes.CDLL(LIB_PATH)
+            vp, i32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+            L.topk_attn_fwd.argtypes = [vp, vp, vp, vp] + [i32] * 9 + [vp]
+            L.topk_attn_fwd_indices.argtypes = [vp, vp, vp, vp] + [i32] * 9 + [vp, vp, vp]
+            L.topk_ffn_fwd.argtypes = [vp, vp, vp, vp] + [i32] * 4 + [vp]
+            L.topk_ffn_fwd_indices.argtypes = [vp, vp, vp, vp] + [i32] * 4 + [vp, vp, vp]
+            L.topk_attn_fwd_host.argtypes = [vp, vp, vp, vp] + [i32] * 9 + [vp]
+            L.topk_ffn_fwd_host.argtypes = [vp, vp, vp, vp] + [i32] * 4 + [vp]
+            L.topk_attn_workspace_bytes.argtypes = [i32] * 8
+            L.topk_attn_workspace_bytes.restype = sz
+            L.topk_ffn_workspace_bytes.argtypes = [i32] * 4
+            L.topk_ffn_workspace_bytes.restype = sz
+            L.topk_check.argtypes = [vp]
+            L.topk_error_string.argtypes = [i32]
+            L.topk_error_string.restype = ctypes.c_char_p
+            L.topk_last_launch_count.argtypes = []
+            L.topk_set_wait_limit_us.argtypes = [ctypes.c_longlong]
+            L.topk_set_wait_limit_us.restype = ctypes.c_longlong
+            L.topk_debug_skip_arrive.argtypes = [i32]
+            for f in ("topk_attn_fwd", "topk_attn_fwd_indices", "topk_ffn_fwd", "topk_ffn_fwd_indices",
+                      "topk_attn_fwd_host", "topk_ffn_fwd_host", "topk_check", "topk_last_launch_count",
+                      "topk_debug_skip_arrive"):
+                getattr(L, f).restype = i32
+            _lib = L
+    return _lib
+
+
+def error_string(code: int) -> str:
+    return lib().topk_error_string(int(code)).decode()
+
+
+def _check(rc: int, where: str) -> None:
+    if rc != 0:
+        raise TopkError(rc, where)
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return TOPK_F32
+    if t.dtype == torch.bfloat16:
+        return TOPK_BF16
+    raise TypeError(f"unsupported dtype {t.dtype}; use float32 or bfloat16")
+
+
+def _ptr(t):
+    return None if t is None else t.data_ptr()
+
+
+def _attn_dims(q, k, v, out):
+    for name, t in (("q", q), ("k", k), ("v", v), ("out", out)):
+        if t.dim() != 4 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous [B, H, L, d] tensor")
+    B, H, Lq, d = q.shape
+    Lk = k.shape[2]
+    if tuple(k.shape) != (B, H, Lk, d) or tuple(v.shape) != (B, H, Lk, d) or tuple(out.shape) != (B, H, Lq, d):
+        raise ValueError("shape mismatch between q, k, v, out")
+    if not (q.dtype == k.dtype == v.dtype == out.dtype):
+        raise TypeError("q, k, v, out must share a dtype")
+    return B, H, Lq, Lk, d
+
+
+def topk_attn_fwd(q, k, v, out, topk: int, chunk: int = 1024, causal: bool = False, stream=None) -> None:
+    """Eq. 4 top-k attention into ``out`` (device tensors [B,H,L,d], fp32 or bf16)."""
+    B, H, Lq, Lk, d = _attn_dims(q, k, v, out)
+    rc = lib().topk_attn_fwd(_ptr(q), _ptr(k), _ptr(v), _ptr(out), B, H, Lq, Lk, d, int(topk), int(chunk),
+                             int(bool(causal)), _dtype_code(q), _stream(stream))
+    _check(rc, "topk_attn_fwd")
+
+
+def topk_attn_fwd_indices(q, k, v, out, topk: int, chunk: int = 1024, causal: bool = False, idx=None,
+                          score=None, stream=None) -> None:
+    """topk_attn_fwd plus kept indices idx [B,H,Lq,topk] int32 and scores [B,H,Lq,topk] fp32."""
+    B, H, Lq, Lk, d = _attn_dims(q, k, v, out)
+    for name, t, dt in (("idx", idx, torch.int32), ("score", score, torch.float32)):
+        if t is not None and (t.dtype != dt or tuple(t.shape) != (B, H, Lq, topk) or not t.is_contiguous()):
+            raise ValueError(f"{name} must be a contiguous [B,H,Lq,topk] {dt} tensor")
+    rc = lib().topk_attn_fwd_indices(_ptr(q), _ptr(k), _ptr(v), _ptr(out), B, H, Lq, Lk, d, int(topk), int(chunk),
+                                     int(bool(causal)), _dtype_code(q), _ptr(idx), _ptr(score), _stream(stream))
+    _check(rc, "topk_attn_fwd_indices")
+
+
+def topk_attn_fwd_host(q, k, v, out, topk: int, chunk: int = 1024, causal: bool = False, stream=None) -> None:
+    """End-to-end call on HOST tensors (pinned is fastest); synchronises the stream."""
+    B, H, Lq, Lk, d = _attn_dims(q, k, v, out)
+    rc = lib().topk_attn_fwd_host(_ptr(q), _ptr(k), _ptr(v), _ptr(out), B, H, Lq, Lk, d, int(topk), int(chunk),
+                                  int(bool(causal)), _dtype_code(q), _stream(stream))
+    _check(rc, "topk_attn_fwd_host")
+
+
+def _ffn_dims(x, W1, W2, out):
+    for name, t in (("x", x), ("W1", W1), ("W2", W2), ("out", out)):
+        if t.dim() != 2 or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous 2-D tensor")
+    N, dm = x.shape
+    dff = W1.shape[0]
+    if tuple(W1.shape) != (dff, dm) or tuple(W2.shape) != (dff, dm) or tuple(out.shape) != (N, dm):
+        raise ValueError("shape mismatch between x, W1, W2, out")
+    if not (x.dtype == W1.dtype == W2.dtype == torch.bfloat16) or out.dtype != torch.float32:
+        raise TypeError("x, W1, W2 must be bfloat16 and out float32")
+    return N, dm, dff
+
+
+def topk_ffn_fwd(x, W1, W2, out, topk: int, stream=None) -> None:
+    """Eq. 3 with top-k: out [N, d_model] fp32 from x [N, d_model], W1/W2 [d_ff, d_model] bf16."""
+    N, dm, dff = _ffn_dims(x, W1, W2, out)
+    rc = lib().topk_ffn_fwd(_ptr(x), _ptr(W1), _ptr(W2), _ptr(out), N, dm, dff, int(topk), _stream(stream))
+    _check(rc, "topk_ffn_fwd")
+
+
+def topk_ffn_fwd_indices(x, W1, W2, out, topk: int, idx=None, score=None, stream=None) -> None:
+    N, dm, dff = _ffn_dims(x, W1, W2, out)
+    rc = lib().topk_ffn_fwd_indices(_ptr(x), _ptr(W1), _ptr(W2), _ptr(out), N, dm, dff, int(topk), _ptr(idx),
+                                    _ptr(score), _stream(stream))
+    _check(rc, "topk_ffn_fwd_indices")
+
+
+def topk_ffn_fwd_host(x, W1, W2, out, topk: int, stream=None) -> None:
+    N, dm, dff = _ffn_dims(x, W1, W2, out)
+    rc = lib().topk_ffn_fwd_host(_ptr(x), _ptr(W1), _ptr(W2), _ptr(out), N, dm, dff, int(topk), _stream(stream))
+    _check(rc, "topk_ffn_fwd_host")
+
+
+def topk_attn_workspace_bytes(B, H, Lq, Lk, d, topk, chunk, dtype) -> int:
+    return int(lib().topk_attn_workspace_bytes(B, H, Lq, Lk, d, topk, chunk, dtype))
+
+
+def topk_ffn_workspace_bytes(N, d_model, d_ff, topk) -> int:
+    return int(lib().topk_ffn_workspace_bytes(N, d_model, d_ff, topk))
+
+
+def topk_check(stream=None) -> None:
+    """Synchronise and raise if a kernel recorded a device-side error since the last check."""
+    _check(lib().topk_check(_stream(stream)), "topk_check")
+
+
+def topk_last_launch_count() -> int:
+    return int(lib().topk_last_launch_count())
+
+
+def topk_set_wait_limit_us(us: int) -> int:
+    return int(lib().topk_set_wait_limit_us(int(us)))
+
+
+# convenience wrappers that allocate the outputs ---------------------------------------------
+
+def attention(q, k, v, topk: int, chunk: int = 1024, causal: bool = False, return_indices: bool = False,
+              stream=None):
+    out = torch.empty_like(q)
+    if not return_indices:
+        topk_attn_fwd(q, k, v, out, topk, chunk, causal, stream)
+        return out
+    B, H, Lq, _ = q.shape
+    idx = torch.empty(B, H, Lq, topk, dtype=torch.int32, device=q.device)
+    score = torch.empty(B, H, Lq, topk, dtype=torch.float32, device=q.device)
+    topk_attn_fwd_indices(q, k, v, out, topk, chunk, causal, idx, score, stream)
+    return out, idx, score
+
+
+def ffn(x, W1, W2, topk: int, return_indices: bool = False, stream=None):
+    out = torch.empty(x.shape[0], x.shape[1], dtype=torch.float32, device=x.device)
+    if not return_indices:
+        topk_ffn_fwd(x, W1, W2, out, topk, stream)
+        return out
+    idx = torch.empty(x.shape[0], topk, dtype=torch.int32, device=x.device)
+    score = torch.empty(x.shape[0], topk, dtype=torch.float32, device=x.device)
+    topk_ffn_fwd_indices(x, W1, W2, out, topk, idx, score, stream)
+    return out, idx, score

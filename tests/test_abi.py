@@ -1,0 +1,67 @@
+"""The C-ABI library loads and exports every symbol include/topk_attention.h declares,
+and rejects bad arguments before launching anything (CPU only: no compute call runs)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2106_06899_gb300 import build
+from paper_2106_06899_gb300 import topk as T
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared():
+    text = open(os.path.join(ROOT, "include", "topk_attention.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(topk_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build_library()
+    return T.lib()
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared()
+    assert "topk_attn_fwd" in names and "topk_ffn_fwd" in names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_error_strings(lib):
+    for code in (0, -1, -2, -3, -4, -5, -6):
+        assert T.error_string(code)
+    assert T.error_string(-99) == "unknown error code"
+
+
+def _attn(lib, **kw):
+    a = dict(q=16, k=16, v=16, out=16, B=1, H=1, Lq=8, Lk=8, d=64, topk=4, chunk=8, causal=0, dtype=1)
+    a.update(kw)
+    return lib.topk_attn_fwd(a["q"], a["k"], a["v"], a["out"], a["B"], a["H"], a["Lq"], a["Lk"], a["d"],
+                             a["topk"], a["chunk"], a["causal"], a["dtype"], None)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(q=None), -1), (dict(out=None), -1), (dict(B=0), -1), (dict(Lk=-1), -1), (dict(topk=0), -1),
+    (dict(topk=9), -1), (dict(chunk=0), -1), (dict(causal=1, Lk=9, topk=2), -1), (dict(causal=2), -1),
+    (dict(dtype=7), -1), (dict(d=96), -2), (dict(dtype=0, d=48), -2), (dict(topk=600, Lk=1000), -2),
+    (dict(q=24), -2),
+])
+def test_attention_argument_errors(lib, kw, code):
+    assert _attn(lib, **kw) == code
+
+
+def test_ffn_argument_errors(lib):
+    f = lib.topk_ffn_fwd
+    assert f(None, 16, 16, 16, 4, 64, 128, 8, None) == -1
+    assert f(16, 16, 16, 16, 4, 64, 128, 0, None) == -1
+    assert f(16, 16, 16, 16, 4, 64, 128, 129, None) == -1
+    assert f(16, 16, 16, 16, 4, 100, 128, 8, None) == -2
+    assert f(16, 16, 16, 16, 4, 64, 4096, 2000, None) == -2
+
+
+def test_attention_needs_no_workspace(lib):
+    assert T.topk_attn_workspace_bytes(1, 12, 65536, 65536, 64, 64, 1024, 1) == 0

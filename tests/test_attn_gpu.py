@@ -1,0 +1,148 @@
+"""GPU parity: top-k attention through the C ABI against the CPU oracle.
+
+Every case runs libtopk.so on cuda:0 and compares, row by row, with the fp64
+oracle under the rules in _parity.py (exact index sets outside near ties,
+validity of every kept key, outputs within 2e-2 for bf16 / 1e-5 for fp32).
+Small shapes are checked on every row; full-size workloads on sampled rows,
+in the launch configuration the benchmark times.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2106_06899_gb300 import topk as T
+from paper_2106_06899_gb300 import workloads as W
+
+from ._parity import check_rows
+
+pytestmark = pytest.mark.gpu
+
+
+def _run(q, k, v, topk, chunk=1024, causal=False):
+    dq, dk, dv = q.cuda(), k.cuda(), v.cuda()
+    out, idx, score = T.attention(dq, dk, dv, topk, chunk, causal, return_indices=True)
+    T.topk_check()
+    d = q.shape[-1]
+    return out.float().cpu().reshape(-1, d), idx.cpu().reshape(-1, topk), score.cpu().reshape(-1, topk)
+
+
+def _check(q, k, v, topk, dtype, rows=None, chunk=1024, causal=False):
+    out, idx, score = _run(q, k, v, topk, chunk, causal)
+    total = q.shape[0] * q.shape[1] * q.shape[2]
+    rows = np.arange(total) if rows is None else np.asarray(rows)
+    return check_rows(q=q, k=k, v=v, rows=rows, gpu_out=out[rows].numpy(), gpu_idx=idx[rows].numpy(),
+                      gpu_score=score[rows].numpy(), topk=topk, dtype=dtype, causal=causal)
+
+
+def _workload(name):
+    w = W.WORKLOADS[name]
+    return w, W.make_inputs(w)
+
+
+def test_tiny_fp32_all_rows():
+    w, (q, k, v) = _workload("tiny_fp32")
+    st = _check(q, k, v, w.topk, "f32", chunk=w.chunk)
+    assert st["rows"] == 512
+
+
+def test_bert_base_all_rows():
+    w, (q, k, v) = _workload("bert_base")
+    st = _check(q, k, v, w.topk, "bf16", chunk=w.chunk)
+    assert st["exact_set_frac"] > 0.5
+
+
+def test_bert_base_all_keys_is_plain_attention():
+    w, (q, k, v) = _workload("bert_base_all_keys")
+    out, idx, score = _run(q, k, v, w.topk, w.chunk)
+    assert torch.equal(idx.sort(dim=1).values, torch.arange(w.Lk, dtype=torch.int32).expand(idx.shape[0], -1))
+    rows = W.sample_rows(w.rows, 2048, seed=5).numpy()
+    ref = oracle.vanilla(q, k, v, rows=rows)
+    assert np.abs(out[rows].numpy() - ref).max() <= 2e-2
+    check_rows(q=q, k=k, v=v, rows=rows, gpu_out=out[rows].numpy(), gpu_idx=idx[rows].numpy(),
+               gpu_score=score[rows].numpy(), topk=w.topk, dtype="bf16")
+
+
+def test_long_65k_sampled_rows():
+    w, (q, k, v) = _workload("long_65k")
+    rows = W.sample_rows(w.rows, 96, seed=2).numpy()
+    st = _check(q, k, v, w.topk, "bf16", rows=rows, chunk=w.chunk)
+    assert st["rows"] == len(rows)
+
+
+def test_causal_16k_sampled_rows():
+    w, (q, k, v) = _workload("causal_16k")
+    L = w.Lq
+    first = np.arange(0, 200)  # rows i < k keep exactly {0..i}
+    pick = W.sample_rows(w.rows, 48, seed=3).numpy()
+    rows = np.unique(np.concatenate([first, L * 17 + first[:40], pick]))
+    out, idx, score = _run(q, k, v, w.topk, w.chunk, causal=True)
+    check_rows(q=q, k=k, v=v, rows=rows, gpu_out=out[rows].numpy(), gpu_idx=idx[rows].numpy(),
+               gpu_score=score[rows].numpy(), topk=w.topk, dtype="bf16", causal=True)
+    for i in range(w.topk):
+        got = idx[i].numpy()
+        assert sorted(got[got >= 0].tolist()) == list(range(i + 1))
+
+
+@pytest.mark.parametrize("dtype,d", [("bf16", 64), ("bf16", 128), ("f32", 64), ("f32", 32)])
+@pytest.mark.parametrize("topk", [1, 17, 64, 128])
+def test_ragged_shapes(dtype, d, topk):
+    # neither length is a multiple of the 128-row query tile or the key tile
+    q, k, v = W.attention_inputs(2, 3, 300, 777, d, dtype=dtype, seed=100 + topk + d)
+    _check(q, k, v, topk, dtype)
+
+
+@pytest.mark.parametrize("dtype,d", [("bf16", 64), ("bf16", 128), ("f32", 64)])
+@pytest.mark.parametrize("topk", [5, 128])
+def test_ragged_causal(dtype, d, topk):
+    q, k, v = W.attention_inputs(1, 3, 650, 650, d, dtype=dtype, seed=200 + topk)
+    _check(q, k, v, topk, dtype, causal=True)
+
+
+@pytest.mark.parametrize("dtype,d,topk", [("bf16", 64, 200), ("bf16", 128, 512), ("f32", 64, 300)])
+def test_large_k(dtype, d, topk):
+    q, k, v = W.attention_inputs(1, 2, 130, 700, d, dtype=dtype, seed=300 + topk)
+    _check(q, k, v, topk, dtype)
+
+
+def test_edge_shapes():
+    # one query, one key, k = Lk, and many tiny heads
+    for (B, H, Lq, Lk, d, topk, dtype) in [(1, 1, 1, 1, 64, 1, "bf16"), (1, 1, 1, 300, 64, 300, "bf16"),
+                                            (3, 5, 7, 9, 64, 9, "bf16"), (2, 2, 129, 257, 128, 3, "bf16"),
+                                            (1, 1, 1, 1, 16, 1, "f32"), (4, 4, 33, 40, 16, 40, "f32")]:
+        q, k, v = W.attention_inputs(B, H, Lq, Lk, d, dtype=dtype, seed=B + H + Lq + Lk)
+        _check(q, k, v, topk, dtype)
+
+
+def test_chunk_does_not_change_results():
+    q, k, v = W.attention_inputs(1, 4, 700, 1500, 64, dtype="bf16", seed=9)
+    outs = [_run(q, k, v, 32, chunk=c) for c in (1, 128, 1000, 4096)]
+    for o in outs[1:]:
+        assert torch.equal(o[0], outs[0][0]) and torch.equal(o[1], outs[0][1])
+
+
+def test_key_permutation_equivariance():
+    q, k, v = W.attention_inputs(1, 2, 256, 1024, 64, dtype="bf16", seed=10)
+    perm = torch.randperm(1024, generator=torch.Generator().manual_seed(4))
+    a_out, a_idx, _ = _run(q, k, v, 16)
+    b_out, b_idx, _ = _run(q, k[:, :, perm].contiguous(), v[:, :, perm].contiguous(), 16)
+    assert torch.equal(a_out, b_out)
+    assert torch.equal(perm[b_idx.long()].int(), a_idx)
+
+
+def test_outputs_fully_written():
+    # outputs pre-filled with NaN must come back finite everywhere
+    q, k, v = W.attention_inputs(2, 2, 333, 500, 64, dtype="bf16", seed=12)
+    dq, dk, dv = q.cuda(), k.cuda(), v.cuda()
+    out = torch.full_like(dq, float("nan"))
+    T.topk_attn_fwd(dq, dk, dv, out, 24)
+    T.topk_check()
+    assert torch.isfinite(out).all()
+
+
+def test_e2e_host_entry_matches_device_entry():
+    q, k, v = W.attention_inputs(1, 2, 300, 600, 64, dtype="bf16", seed=13)
+    dev = T.attention(q.cuda(), k.cuda(), v.cuda(), 32).cpu()
+    host_out = torch.empty_like(q).pin_memory()
+    T.topk_attn_fwd_host(q.pin_memory(), k.pin_memory(), v.pin_memory(), host_out, 32)
+    assert torch.equal(host_out, dev)
