@@ -46,7 +46,12 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU work budget of the oracle baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-clocks", action="store_true")
-    return p.parse_args()
+    p.add_argument("--kernel-only", action="store_true",
+                   help="time the device call only: no end-to-end leg, clocks or CPU baseline (profiling)")
+    a = p.parse_args()
+    if a.kernel_only:
+        a.no_clocks, a.no_cpu_baseline, a.e2e_steps = True, True, 0
+    return a
 
 
 def peaks():
@@ -291,24 +296,27 @@ def run_ours(args):
     value = world * w.tokens / (ms_max / 1e3)
 
     # end to end through the host-buffer C-ABI entry: H2D copies, call, D2H copy, every step
-    pinned = [t.pin_memory() for t in host]
-    hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
-    if w.kind == "ffn":
-        def e2e_step():
-            T.topk_ffn_fwd_host(pinned[0], pinned[1], pinned[2], hout, w.topk)
-    else:
-        def e2e_step():
-            T.topk_attn_fwd_host(pinned[0], pinned[1], pinned[2], hout, w.topk, w.chunk, w.causal)
-    e2e_step()
-    barrier()
-    t0 = time.perf_counter()
-    for _ in range(args.e2e_steps):
+    e2e = None
+    if args.e2e_steps > 0:
+        pinned = [t.pin_memory() for t in host]
+        hout = torch.empty(out.shape, dtype=out.dtype).pin_memory()
+        if w.kind == "ffn":
+            def e2e_step():
+                T.topk_ffn_fwd_host(pinned[0], pinned[1], pinned[2], hout, w.topk)
+        else:
+            def e2e_step():
+                T.topk_attn_fwd_host(pinned[0], pinned[1], pinned[2], hout, w.topk, w.chunk, w.causal)
         e2e_step()
-    e2e_s = (time.perf_counter() - t0) / args.e2e_steps
-    te = torch.tensor([e2e_s], device="cuda")
-    if world > 1:
-        dist.all_reduce(te, op=dist.ReduceOp.MAX)
-    e2e_value = world * w.tokens / float(te.item())
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(args.e2e_steps):
+            e2e_step()
+        e2e_s = (time.perf_counter() - t0) / args.e2e_steps
+        te = torch.tensor([e2e_s], device="cuda")
+        if world > 1:
+            dist.all_reduce(te, op=dist.ReduceOp.MAX)
+        e2e = {"value": world * w.tokens / float(te.item()), "unit": "tokens/s", "h2d_bytes_per_step": in_bytes,
+               "d2h_bytes_per_step": out.numel() * out.element_size()}
 
     pk = peaks()
     flops = work_flops(w)
@@ -323,8 +331,7 @@ def run_ours(args):
                      "frac": achieved / pk["bf16"], "traffic": None,
                      "peak_source": f"{pk['source']} bf16 dense (burst)",
                      "kernel": "attn_tc_kernel" if w.kind == "attn" else "ffn kernels"},
-        "e2e": {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": in_bytes,
-                "d2h_bytes_per_step": out.numel() * out.element_size()},
+        "e2e": e2e,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clocks,
     }

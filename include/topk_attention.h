@@ -102,6 +102,7 @@ int topk_attn_fwd_indices(const void* q, const void* k, const void* v, void* out
  *   W2 : [d_ff, d_model] bf16; row j is value j.
  *   out: [N, d_model] fp32 device pointer.
  *   d_model: a multiple of 64, at most 4096.  1 <= topk <= d_ff, topk <= 1024.
+ *   Scratch: topk_ffn_workspace_bytes(); it grows linearly with N.
  * Top-k is taken over the signed scores; ReLU is applied after selection.
  */
 int topk_ffn_fwd(const void* x, const void* W1, const void* W2, void* out, int N, int d_model, int d_ff,

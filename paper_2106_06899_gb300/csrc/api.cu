@@ -201,6 +201,21 @@ size_t topk_ffn_workspace_bytes(int N, int d_model, int d_ff, int topk) {
   return ffn_workspace_bytes(N, d_model, d_ff, topk);
 }
 
+namespace {
+// After a synchronising host-buffer call: report any device-side error flag.
+int host_call_status(int rc) {
+  if (rc != TOPK_OK) return rc;
+  DeviceState* dev = device_state();
+  if (!dev) return TOPK_ERR_NO_DEVICE;
+  unsigned word = 0;
+  if (cudaMemcpy(&word, dev->error_word, sizeof word, cudaMemcpyDeviceToHost) != cudaSuccess) return TOPK_ERR_CUDA;
+  if (!word) return TOPK_OK;
+  const unsigned zero = 0;
+  cudaMemcpy(dev->error_word, &zero, sizeof zero, cudaMemcpyHostToDevice);
+  return (word & kDevErrTimeout) ? TOPK_ERR_TIMEOUT : TOPK_ERR_WORKSPACE;
+}
+}  // namespace
+
 int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk, int d,
                        int topk, int chunk, int causal, int dtype, void* stream) {
   if (!q || !k || !v || !out) return TOPK_ERR_INVALID_ARG;
@@ -232,7 +247,7 @@ int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, i
   if (dout) cudaFreeAsync(dout, st);
   if (cudaStreamSynchronize(st) != cudaSuccess && rc == TOPK_OK) rc = TOPK_ERR_CUDA;
   t_last_launches = launches;
-  return rc;
+  return host_call_status(rc);
 }
 
 int topk_ffn_fwd_host(const void* x, const void* W1, const void* W2, void* out, int N, int d_model, int d_ff,
@@ -265,7 +280,7 @@ int topk_ffn_fwd_host(const void* x, const void* W1, const void* W2, void* out, 
   if (dout) cudaFreeAsync(dout, st);
   if (cudaStreamSynchronize(st) != cudaSuccess && rc == TOPK_OK) rc = TOPK_ERR_CUDA;
   t_last_launches = launches;
-  return rc;
+  return host_call_status(rc);
 }
 
 int topk_check(void* stream) {

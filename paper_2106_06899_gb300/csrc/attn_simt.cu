@@ -16,7 +16,8 @@ namespace topk {
 
 namespace {
 
-constexpr int KT = 32;  // keys per staged tile
+constexpr int KT = 32;    // keys per staged tile
+constexpr int GROUPS = 8;  // pending score groups per row
 
 template <typename T>
 __device__ __forceinline__ float to_f32(T x);
@@ -36,7 +37,7 @@ __global__ void __launch_bounds__(ROWS) attn_simt_kernel(const T* __restrict__ q
                                                          int32_t* __restrict__ idx, float* __restrict__ score) {
   extern __shared__ __align__(16) uint8_t smem_raw[];
   float* ks = reinterpret_cast<float*>(smem_raw);                       // [KT][D]
-  uint64_t* heap_mem = reinterpret_cast<uint64_t*>(smem_raw + KT * D * sizeof(float));  // [topk][ROWS]
+  uint8_t* sel_mem = smem_raw + KT * D * sizeof(float);  // heap [topk][ROWS], records [GROUPS][ROWS]
 
   const int n_qt = (Lq + ROWS - 1) / ROWS;
   const int unit = blockIdx.x;
@@ -55,7 +56,7 @@ __global__ void __launch_bounds__(ROWS) attn_simt_kernel(const T* __restrict__ q
   }
 
   RowHeap<ROWS> heap;
-  heap.init(heap_mem, tid, topk);
+  heap.init(sel_mem, tid, topk, GROUPS);
 
   const int kend = causal ? min(Lk, (qt + 1) * ROWS) : Lk;
   const uint32_t lim = static_cast<uint32_t>(causal ? min(i + 1, Lk) : Lk);
@@ -83,21 +84,21 @@ __global__ void __launch_bounds__(ROWS) attn_simt_kernel(const T* __restrict__ q
         s[e] = fmaf(qr[t + 3], kv.w, s[e]);
       }
     }
-    if (j0 + KT > cta_lim_min) mask32(s, static_cast<uint32_t>(j0), lim);
-    heap.offer32(s, static_cast<uint32_t>(j0));
+    if (j0 + KT > cta_lim_min) mask_scores(s, static_cast<uint32_t>(j0), lim);
+    heap.offer(s, static_cast<uint32_t>(j0));
   }
 
+  heap.finish();  // every lane takes part (warp-synchronous flush)
   if (!row_ok) return;
-  heap.sort_desc();
   const size_t orow = static_cast<size_t>(bh) * Lq + i;
-  softmax_gather_store<T, D, ROWS>(heap, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
+  softmax_gather_store<T, D>(heap, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
   if (idx || score)
     write_selection(heap, idx ? idx + orow * topk : nullptr, score ? score + orow * topk : nullptr);
 }
 
 template <typename T, int D, int ROWS>
 int launch_simt(const AttnArgs& a, cudaStream_t st) {
-  const size_t smem = static_cast<size_t>(KT) * D * sizeof(float) + static_cast<size_t>(a.topk) * ROWS * 8;
+  const size_t smem = static_cast<size_t>(KT) * D * sizeof(float) + RowHeap<ROWS>::bytes(a.topk, GROUPS);
   auto kern = attn_simt_kernel<T, D, ROWS>;
   if (smem > 48 * 1024) {
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=

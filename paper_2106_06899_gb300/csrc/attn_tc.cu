@@ -40,9 +40,11 @@ struct TcShape<64> {
 };
 template <>
 struct TcShape<128> {
-  static constexpr int N = 128;
-  static constexpr int S = 2;
+  static constexpr int N = 64;
+  static constexpr int S = 3;
 };
+
+using Sel = RowHeap<BM>;
 
 template <int D>
 struct Layout {
@@ -53,10 +55,21 @@ struct Layout {
   static constexpr uint32_t KST_BYTES = N * D * 2;
   static constexpr size_t OFF_Q = 0;
   static constexpr size_t OFF_K = OFF_Q + Q_BYTES;
-  static constexpr size_t OFF_HEAP = OFF_K + static_cast<size_t>(S) * KST_BYTES;
+  static constexpr size_t OFF_SEL = OFF_K + static_cast<size_t>(S) * KST_BYTES;
   static constexpr int NBARS = 2 * S + 7;
   static constexpr size_t CTRL_BYTES = 256;
-  static size_t bytes(int topk) { return 1024 + OFF_HEAP + static_cast<size_t>(topk) * BM * 8 + CTRL_BYTES; }
+  static constexpr size_t kMaxSmem = 232448;
+  static constexpr size_t kFixed = 1024 + OFF_SEL + CTRL_BYTES;
+
+  // pending score groups per row: as many as fit, at most 24 (0: the heap does not fit)
+  static int rec_cap(int topk) {
+    const size_t heap = static_cast<size_t>(topk) * BM * 8;
+    if (kFixed + heap + Sel::bytes(0, 4) >= kMaxSmem) return 0;
+    const size_t room = (kMaxSmem - kFixed - heap) / (BM * 36);
+    return room >= 24 ? 24 : static_cast<int>(room);
+  }
+  __host__ __device__ static size_t sel_bytes(int topk, int gr) { return (Sel::bytes(topk, gr) + 15) & ~size_t(15); }
+  static size_t bytes(int topk) { return kFixed + sel_bytes(topk, rec_cap(topk)); }
 };
 
 // Waits on an mbarrier phase with lane 0 of the warp and broadcasts the
@@ -85,8 +98,8 @@ template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmk,
                    const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ out, int BH, int Lq, int Lk,
-                   int topk, int causal, int n_units, int32_t* __restrict__ idx, float* __restrict__ score,
-                   DevCtl ctl) {
+                   int topk, int rec_cap, int causal, int n_units, int32_t* __restrict__ idx,
+                   float* __restrict__ score, DevCtl ctl) {
   using L = Layout<D>;
   constexpr int N = L::N, S = L::S, R = L::R;
   constexpr uint32_t IDESC = idesc_bf16_f32(BM, N);
@@ -96,8 +109,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint8_t* q_s = smem + L::OFF_Q;
   uint8_t* k_s = smem + L::OFF_K;
-  uint64_t* heap_mem = reinterpret_cast<uint64_t*>(smem + L::OFF_HEAP);
-  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + L::OFF_HEAP + static_cast<size_t>(topk) * BM * 8);
+  uint8_t* sel_mem = smem + L::OFF_SEL;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(sel_mem + L::sel_bytes(topk, rec_cap));
   uint64_t* full_k = bars;
   uint64_t* empty_k = bars + S;
   uint64_t* q_full = bars + 2 * S;
@@ -254,13 +267,13 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int row = quad * 32 + lane;
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
     uint32_t acc_it = 0;
-    RowHeap<BM> heap;
+    Sel heap;
     bool ok = true;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
       int bh, qt;
       decode(u, bh, qt);
       const int i_row = qt * BM + row;
-      heap.init(heap_mem, row, topk);
+      heap.init(sel_mem, row, topk, rec_cap);
       const int nk = key_tiles(qt);
       const uint32_t lim = static_cast<uint32_t>(causal ? min(i_row + 1, Lk) : Lk);
       const int lim_min = causal ? min(qt * BM + 1, Lk) : Lk;
@@ -274,26 +287,26 @@ __global__ void __launch_bounds__(kThreads, 1)
         const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(b * N);
         const uint32_t jt = static_cast<uint32_t>(kt * N);
 #pragma unroll 1
-        for (int c = 0; c < N / 32; ++c) {
-          float vals[32];
+        for (int c = 0; c < N / 64; ++c) {
+          float vals[64];
           __syncwarp();
-          tmem_ld32(taddr + c * 32, vals);
+          tmem_ld64(taddr + c * 64, vals);
           tmem_wait_ld();
-          if (c == N / 32 - 1) {
+          if (c == N / 64 - 1) {
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&acc_empty[b]);
           }
-          const uint32_t j0 = jt + static_cast<uint32_t>(c * 32);
-          if (static_cast<int>(j0) + 32 > lim_min) mask32(vals, j0, lim);
-          heap.offer32(vals, j0);
+          const uint32_t j0 = jt + static_cast<uint32_t>(c * 64);
+          if (static_cast<int>(j0) + 64 > lim_min) mask_scores(vals, j0, lim);
+          heap.offer(vals, j0);
         }
       }
       if (!ok) break;
+      heap.finish();  // every lane takes part (warp-synchronous flush)
       if (i_row < Lq) {
-        heap.sort_desc();
         const size_t orow = static_cast<size_t>(bh) * Lq + i_row;
-        softmax_gather_store<__nv_bfloat16, D, BM>(heap, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
+        softmax_gather_store<__nv_bfloat16, D>(heap, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
         if (idx || score)
           write_selection(heap, idx ? idx + orow * topk : nullptr, score ? score + orow * topk : nullptr);
       }
@@ -319,15 +332,16 @@ int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st
   const int n_units = BH * ((a.Lq + BM - 1) / BM);
   // At least 120 KB so that a second CTA never shares the SM: each CTA takes
   // all TMEM columns it needs for its whole (persistent) lifetime.
-  const size_t smem = L::bytes(a.topk) > 120 * 1024 ? L::bytes(a.topk) : 120 * 1024;
+  const size_t need = L::bytes(a.topk);
+  const size_t smem = need > 120 * 1024 ? need : 120 * 1024;
   auto kern = attn_tc_kernel<D>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
       cudaSuccess)
     return -1;
   const int grid = n_units < num_sms ? n_units : num_sms;
   kern<<<grid, kThreads, smem, st>>>(tmq, tmk, static_cast<const __nv_bfloat16*>(a.v),
-                                     static_cast<__nv_bfloat16*>(a.out), BH, a.Lq, a.Lk, a.topk, a.causal, n_units,
-                                     a.idx, a.score, ctl);
+                                     static_cast<__nv_bfloat16*>(a.out), BH, a.Lq, a.Lk, a.topk,
+                                     L::rec_cap(a.topk), a.causal, n_units, a.idx, a.score, ctl);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
@@ -335,8 +349,8 @@ int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st
 
 bool attn_tc_supports(const AttnArgs& a) {
   if (a.dtype != 1 || a.topk > kTcMaxK) return false;
-  if (a.d == 64) return Layout<64>::bytes(a.topk) <= 232448;
-  if (a.d == 128) return Layout<128>::bytes(a.topk) <= 232448;
+  if (a.d == 64) return Layout<64>::rec_cap(a.topk) >= 4;
+  if (a.d == 128) return Layout<128>::rec_cap(a.topk) >= 4;
   return false;
 }
 

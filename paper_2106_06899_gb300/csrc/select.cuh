@@ -10,7 +10,7 @@
 //
 // Each row owns a min-heap of its k best keys in shared memory, laid out
 // [slot][row] so that the 32 threads of a warp always touch 32 different
-// banks whatever slots they visit.  Scores stream in by ascending key index,
+// banks whatever slots they visit (128 rows: a 64-bit slot row is 1 KB).  Scores stream in by ascending key index,
 // so a new score can only enter when it is strictly greater than the score
 // at the heap root (an equal score has a larger index and ranks lower);
 // `tau` caches that root score (-inf while the heap is not yet full) and
@@ -41,20 +41,50 @@ __device__ __forceinline__ float key_score(uint64_t key) { return unord_f32(stat
 
 __device__ __forceinline__ uint32_t key_index(uint64_t key) { return ~static_cast<uint32_t>(key); }
 
-// Exact per-row top-k (min-heap of packed keys) in shared memory.
-// ROWS = number of rows sharing the [slot][row] array (the row stride).
+// Exact per-row top-k: a 4-ary min-heap of packed keys in shared memory,
+// fed through a per-row buffer of pending score groups.
+//
+// The filter compares the maximum of each group of 8 scores with tau (the
+// heap root's score, -inf until the heap is full) and, if it wins, copies
+// the whole group (8 scores and its first key index) into the row's record
+// buffer with two vector stores: no per-element work and no loop on the
+// divergent path.  When any lane of the warp has filled its record buffer,
+// the whole warp expands its records into the heaps in lockstep (flush):
+// elements are offered in ascending key index, each one that beats the
+// current root replaces it.  tau only rises, so records taken against a
+// stale tau can hold a few elements that no longer qualify; they are
+// re-checked at expansion.  The 4-ary heap halves the dependent shared
+// memory round trips of a replace (log4 k levels of four independent loads).
+// ROWS = number of rows sharing the [slot][row] arrays (the row stride);
+// every call of offer*/flush/finish must be made by all 32 lanes of a warp.
 template <int ROWS>
 struct RowHeap {
   uint64_t* base;  // &heap[slot 0][this row]
+  float4* rlo;     // &records_lo[0][this row]: scores 0..3
+  float4* rhi;     // &records_hi[0][this row]: scores 4..7
+  uint32_t* rj;    // &records_j0[0][this row]
   int k;           // capacity
   int n;           // entries filled
+  int rc;          // records pending
+  int gr;          // record capacity
   uint64_t root;   // heap[0] once full
   float tau;       // score of heap[0] once full, else -inf
 
-  __device__ __forceinline__ void init(uint64_t* smem, int row, int cap) {
-    base = smem + row;
+  // shared memory: heap k x ROWS x 8 bytes, then records gr x ROWS x 36 bytes
+  __host__ __device__ static constexpr size_t bytes(int k_, int gr_) {
+    return static_cast<size_t>(ROWS) * (static_cast<size_t>(k_) * 8 + static_cast<size_t>(gr_) * 36);
+  }
+
+  __device__ __forceinline__ void init(uint8_t* smem, int row, int cap, int rec_cap) {
+    base = reinterpret_cast<uint64_t*>(smem) + row;
+    uint8_t* r = smem + static_cast<size_t>(cap) * ROWS * 8;
+    rlo = reinterpret_cast<float4*>(r) + row;
+    rhi = reinterpret_cast<float4*>(r + static_cast<size_t>(rec_cap) * ROWS * 16) + row;
+    rj = reinterpret_cast<uint32_t*>(r + static_cast<size_t>(rec_cap) * ROWS * 32) + row;
     k = cap;
+    gr = rec_cap;
     n = 0;
+    rc = 0;
     root = 0;
     tau = -INFINITY;
   }
@@ -62,22 +92,33 @@ struct RowHeap {
   __device__ __forceinline__ uint64_t get(int p) const { return base[p * ROWS]; }
   __device__ __forceinline__ void put(int p, uint64_t x) { base[p * ROWS] = x; }
 
-  // Sift x down from slot p within a heap of m entries.
+  // Sift x down from slot p within a heap of m entries (children 4p+1..4p+4).
   __device__ __forceinline__ void sift_down(uint64_t x, int p, int m) {
     for (;;) {
-      int c = 2 * p + 1;
+      const int c = 4 * p + 1;
       if (c >= m) break;
       uint64_t a = get(c);
-      if (c + 1 < m) {
-        const uint64_t b = get(c + 1);
-        if (b < a) {
-          a = b;
-          ++c;
+      int ca = c;
+      if (c + 3 < m) {
+        const uint64_t b1 = get(c + 1), b2 = get(c + 2), b3 = get(c + 3);
+        const uint64_t m01 = b1 < a ? b1 : a;
+        const int i01 = b1 < a ? c + 1 : c;
+        const uint64_t m23 = b3 < b2 ? b3 : b2;
+        const int i23 = b3 < b2 ? c + 3 : c + 2;
+        a = m23 < m01 ? m23 : m01;
+        ca = m23 < m01 ? i23 : i01;
+      } else {
+        for (int q = c + 1; q < m; ++q) {
+          const uint64_t b = get(q);
+          if (b < a) {
+            a = b;
+            ca = q;
+          }
         }
       }
       if (a >= x) break;
       put(p, a);
-      p = c;
+      p = ca;
     }
     put(p, x);
   }
@@ -86,7 +127,7 @@ struct RowHeap {
     if (n < k) {
       int c = n;
       while (c > 0) {
-        const int p = (c - 1) >> 1;
+        const int p = (c - 1) >> 2;
         const uint64_t pk = get(p);
         if (pk <= x) break;
         put(c, pk);
@@ -104,29 +145,58 @@ struct RowHeap {
     }
   }
 
-  // Offer 32 scores whose key indices are j0 .. j0+31 (ascending).  Groups
-  // of 8 are tested against tau through their maximum first; only a group
-  // that beats tau is looked at element by element.
-  __device__ __forceinline__ void offer32(const float (&v)[32], uint32_t j0) {
-#pragma unroll
-    for (int g = 0; g < 4; ++g) {
-      const float m = max3f(max3f(v[8 * g], v[8 * g + 1], v[8 * g + 2]),
-                            max3f(v[8 * g + 3], v[8 * g + 4], v[8 * g + 5]), fmaxf(v[8 * g + 6], v[8 * g + 7]));
-      if (m > tau) {
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          if (v[8 * g + e] > tau) push(make_key(v[8 * g + e], j0 + 8 * g + e));
+  // Expand every lane's pending records into its heap, lanes in lockstep.
+  // For each record slot every lane forms the mask of its elements that
+  // still beat tau; then the warp pushes one element per lane per step, so
+  // that one push body serves all lanes at once.  Not inlined: it is the
+  // rare path of every unrolled offer8.
+  __device__ __noinline__ void flush() {
+    const int mxr = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(rc));
+    for (int i = 0; i < mxr; ++i) {
+      unsigned msk = 0;
+      uint32_t j0 = 0;
+      const float* sc = reinterpret_cast<const float*>(rlo + i * ROWS);  // scores 0..3, then 4..7 in rhi
+      if (i < rc) {
+        const float4 a = rlo[i * ROWS];
+        const float4 b = rhi[i * ROWS];
+        j0 = rj[i * ROWS];
+        msk = (a.x > tau ? 1u : 0u) | (a.y > tau ? 2u : 0u) | (a.z > tau ? 4u : 0u) | (a.w > tau ? 8u : 0u) |
+              (b.x > tau ? 16u : 0u) | (b.y > tau ? 32u : 0u) | (b.z > tau ? 64u : 0u) | (b.w > tau ? 128u : 0u);
+      }
+      while (__any_sync(0xffffffffu, msk != 0)) {
+        if (msk) {
+          const int e = __ffs(msk) - 1;
+          msk &= msk - 1;
+          const float v = e < 4 ? sc[e] : reinterpret_cast<const float*>(rhi + i * ROWS)[e - 4];
+          if (v > tau) push(make_key(v, j0 + e));
         }
       }
     }
+    rc = 0;
   }
 
-  // Heap-sort in place: afterwards slots 0 .. n-1 hold the kept keys in
-  // selection order (best first).
-  __device__ __forceinline__ void sort_desc() {
-    if (n < k) {
-      // not full: it is still a valid min-heap of n entries
+  // Offer 8 scores with key indices j0 .. j0+7 (ascending).
+  __device__ __forceinline__ void offer8(const float* v, uint32_t j0) {
+    const float m = max3f(max3f(v[0], v[1], v[2]), max3f(v[3], v[4], v[5]), fmaxf(v[6], v[7]));
+    if (m > tau) {
+      rlo[rc * ROWS] = make_float4(v[0], v[1], v[2], v[3]);
+      rhi[rc * ROWS] = make_float4(v[4], v[5], v[6], v[7]);
+      rj[rc * ROWS] = j0;
+      ++rc;
     }
+    if (__any_sync(0xffffffffu, rc == gr)) flush();
+  }
+
+  template <int W>
+  __device__ __forceinline__ void offer(const float (&v)[W], uint32_t j0) {
+#pragma unroll
+    for (int g = 0; g < W / 8; ++g) offer8(&v[8 * g], j0 + 8 * g);
+  }
+
+  // After the last key: merge what is pending, then heap-sort in place so
+  // that slots 0 .. n-1 hold the kept keys in selection order (best first).
+  __device__ __forceinline__ void finish() {
+    flush();
     for (int m = n - 1; m > 0; --m) {
       const uint64_t x = get(m);
       put(m, get(0));
@@ -136,9 +206,10 @@ struct RowHeap {
 };
 
 // Replace scores of invalid keys (index >= lim) by -inf.
-__device__ __forceinline__ void mask32(float (&v)[32], uint32_t j0, uint32_t lim) {
+template <int W>
+__device__ __forceinline__ void mask_scores(float (&v)[W], uint32_t j0, uint32_t lim) {
 #pragma unroll
-  for (int e = 0; e < 32; ++e)
+  for (int e = 0; e < W; ++e)
     if (j0 + static_cast<uint32_t>(e) >= lim) v[e] = -INFINITY;
 }
 
@@ -167,8 +238,8 @@ __device__ __forceinline__ uint4 f32x8_to_bf16(const float (&f)[8]) {
 // type T (float or bf16) starting at `vbase` (row j at vbase + j * D); the
 // result is written to `orow` (D elements of T).  Accumulation is fp32 over
 // 64-column slices so that at most 64 accumulators are live.
-template <typename T, int D, int ROWS>
-__device__ __forceinline__ void softmax_gather_store(const RowHeap<ROWS>& h, const T* __restrict__ vbase,
+template <typename T, int D, typename Sel>
+__device__ __forceinline__ void softmax_gather_store(const Sel& h, const T* __restrict__ vbase,
                                                      T* __restrict__ orow) {
   constexpr int SL = D < 64 ? D : 64;
   const int n = h.n;
@@ -223,8 +294,8 @@ __device__ __forceinline__ void softmax_gather_store(const RowHeap<ROWS>& h, con
 }
 
 // Debug/parity output: kept indices and fp32 scores in selection order.
-template <int ROWS>
-__device__ __forceinline__ void write_selection(const RowHeap<ROWS>& h, int32_t* idx_row, float* score_row) {
+template <typename Sel>
+__device__ __forceinline__ void write_selection(const Sel& h, int32_t* idx_row, float* score_row) {
   for (int t = 0; t < h.k; ++t) {
     const bool have = t < h.n;
     const uint64_t key = have ? h.get(t) : 0;

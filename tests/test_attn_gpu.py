@@ -146,3 +146,26 @@ def test_e2e_host_entry_matches_device_entry():
     host_out = torch.empty_like(q).pin_memory()
     T.topk_attn_fwd_host(q.pin_memory(), k.pin_memory(), v.pin_memory(), host_out, 32)
     assert torch.equal(host_out, dev)
+
+
+def test_memory_is_linear_in_keys():
+    # Sec. 2.2: memory O(C L_K) for a fixed chunk; here the kernel holds no per-call device scratch at
+    # all, so the peak is the inputs and outputs themselves, linear in L_K
+    peaks = []
+    for Lk in (8192, 16384, 32768, 65536):
+        q, k, v = W.attention_inputs(1, 4, 1024, Lk, 64, dtype="bf16", seed=Lk)
+        torch.cuda.synchronize()
+        torch.cuda.empty_cache()
+        torch.cuda.reset_peak_memory_stats()
+        base = torch.cuda.memory_allocated()
+        free0 = torch.cuda.mem_get_info()[0]
+        dq, dk, dv = q.cuda(), k.cuda(), v.cuda()
+        out = torch.empty_like(dq)
+        T.topk_attn_fwd(dq, dk, dv, out, 64, 1024)
+        T.topk_check()
+        peaks.append(torch.cuda.max_memory_allocated() - base)
+        assert torch.cuda.mem_get_info()[0] >= free0 - (dq.numel() * 2 * 4 + (64 << 20))
+        assert T.topk_attn_workspace_bytes(1, 4, 1024, Lk, 64, 64, 1024, 1) == 0
+        del dq, dk, dv, out
+    d = np.diff(peaks)
+    assert np.allclose(d[1:] / d[:-1], 2.0, rtol=0.02), peaks
