@@ -65,7 +65,9 @@ enum {
   TOPK_ERR_WORKSPACE = -5,   /* a per-row candidate list ran out of room (needs
                                 more keys tied within one bf16 step of the k-th
                                 score than the list holds); outputs invalid */
-  TOPK_ERR_NO_DEVICE = -6    /* no usable sm_103 device */
+  TOPK_ERR_NO_DEVICE = -6,   /* no usable sm_103 device */
+  TOPK_ERR_SCRATCH_LIMIT = -7 /* the problem needs more scratch than the fixed buffer of
+                                 topk_ffn_fwd_noalloc holds */
 };
 
 /*
@@ -111,6 +113,32 @@ int topk_ffn_fwd(const void* x, const void* W1, const void* W2, void* out, int N
 /* topk_ffn_fwd plus the kept indices [N, topk] int32 and scores [N, topk] fp32. */
 int topk_ffn_fwd_indices(const void* x, const void* W1, const void* W2, void* out, int N, int d_model,
                          int d_ff, int topk, int32_t* idx, float* score, void* stream);
+
+/*
+ * topk_ffn_fwd without any device allocation.  The paper has no counterpart:
+ * this entry exists for callers that cannot allocate device memory when they
+ * call -- for instance a host runtime that hands out all device memory from
+ * its own arena and allows no other allocation, or a latency-bound serving
+ * loop that must never wait on an allocator or fail on a fragmented pool.
+ * Instead of taking scratch from the stream-ordered pool it uses one buffer
+ * of TOPK_FFN_NOALLOC_SCRATCH_BYTES that is part of the library: every GPU
+ * that loads libtopk.so holds it until the process exits.
+ *   - Arguments, layouts and results are those of topk_ffn_fwd; the caller
+ *     still passes (and owns) x, W1, W2 and out.
+ *   - Returns TOPK_ERR_SCRATCH_LIMIT, before launching anything, when
+ *     topk_ffn_workspace_bytes() of the arguments exceeds the buffer.
+ *   - The first call on a device looks up the buffer's device address (one
+ *     runtime query, no allocation); make that first call before any stream
+ *     capture on that device.
+ *   - All calls on a device share the one buffer, and each call re-clears
+ *     the parts that must start at zero.  Calls whose work overlaps on the
+ *     GPU (other streams, or other threads) race on the buffer: serialise
+ *     them, e.g. by issuing them on one stream.
+ * It calls no cudaMalloc, cudaFree or other allocating routine.
+ */
+#define TOPK_FFN_NOALLOC_SCRATCH_BYTES (32u << 20)
+int topk_ffn_fwd_noalloc(const void* x, const void* W1, const void* W2, void* out, int N, int d_model,
+                         int d_ff, int topk, void* stream);
 
 /* Bytes of stream-ordered scratch the calls above take for these arguments
  * (0 if none).  Returns 0 as well when the arguments are invalid. */

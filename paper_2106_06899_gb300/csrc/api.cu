@@ -9,7 +9,7 @@
 #include <cstring>
 #include <mutex>
 
-#include "../../include/topk_attention.h"
+#include "topk_attention.h"
 #include "kernels.h"
 
 namespace topk {
@@ -283,6 +283,61 @@ int topk_ffn_fwd_host(const void* x, const void* W1, const void* W2, void* out, 
   return host_call_status(rc);
 }
 
+}  // extern "C"
+
+// ---------------------------------------------------------------- no-allocation FF entry
+namespace topk {
+namespace {
+
+// Scratch of topk_ffn_fwd_noalloc: part of the module image, held by every
+// device that loads the library until the process exits.
+static __device__ __align__(256) unsigned char g_ffn_noalloc_scratch[TOPK_FFN_NOALLOC_SCRATCH_BYTES];
+
+struct NoAllocState {
+  std::once_flag once;
+  void* ptr = nullptr;
+};
+NoAllocState g_noalloc[kMaxDevices];
+
+// Device address of the scratch array on the current device (looked up once
+// per device, with that device current).  Host code must not use the array's
+// name as an address: on the host it is only a stand-in for the symbol.
+void* noalloc_scratch() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  NoAllocState& s = g_noalloc[dev];
+  std::call_once(s.once, [&s]() {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_ffn_noalloc_scratch) == cudaSuccess) s.ptr = p;
+  });
+  return s.ptr;
+}
+
+}  // namespace
+}  // namespace topk
+
+extern "C" {
+
+int topk_ffn_fwd_noalloc(const void* x, const void* W1, const void* W2, void* out, int N, int d_model, int d_ff,
+                         int topk, void* stream) {
+  FfnArgs a{x, W1, W2, static_cast<float*>(out), N, d_model, d_ff, topk, nullptr, nullptr, nullptr, 0};
+  int rc = validate_ffn(a);
+  if (rc) return rc;
+  DeviceState* dev = device_state();
+  if (!dev) return TOPK_ERR_NO_DEVICE;
+  if (dev->cc_major != 10 || dev->cc_minor != 3) return TOPK_ERR_NO_DEVICE;
+  if (ffn_workspace_bytes(N, d_model, d_ff, topk) > TOPK_FFN_NOALLOC_SCRATCH_BYTES) return TOPK_ERR_SCRATCH_LIMIT;
+  void* scratch = noalloc_scratch();
+  if (!scratch) return TOPK_ERR_CUDA;
+  a.workspace = scratch;
+  a.workspace_bytes = TOPK_FFN_NOALLOC_SCRATCH_BYTES;
+  const int n = ffn_tc(a, make_ctl(dev), dev->num_sms, static_cast<cudaStream_t>(stream));
+  if (n == 0) return TOPK_ERR_UNSUPPORTED;
+  if (n < 0) return TOPK_ERR_CUDA;
+  t_last_launches = n;
+  return TOPK_OK;
+}
+
 int topk_check(void* stream) {
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   if (cudaStreamSynchronize(st) != cudaSuccess) return TOPK_ERR_CUDA;
@@ -309,6 +364,7 @@ const char* topk_error_string(int code) {
     case TOPK_ERR_TIMEOUT: return "device pipeline wait timed out; outputs invalid";
     case TOPK_ERR_WORKSPACE: return "per-row candidate list overflowed; outputs invalid";
     case TOPK_ERR_NO_DEVICE: return "no usable sm_103 device";
+    case TOPK_ERR_SCRATCH_LIMIT: return "problem needs more scratch than the fixed no-allocation buffer holds";
     default: return "unknown error code";
   }
 }

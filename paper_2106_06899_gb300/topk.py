@@ -44,6 +44,7 @@ def lib() -> ctypes.CDLL:
             L.topk_ffn_fwd_indices.argtypes = [vp, vp, vp, vp] + [i32] * 4 + [vp, vp, vp]
             L.topk_attn_fwd_host.argtypes = [vp, vp, vp, vp] + [i32] * 9 + [vp]
             L.topk_ffn_fwd_host.argtypes = [vp, vp, vp, vp] + [i32] * 4 + [vp]
+            L.topk_ffn_fwd_noalloc.argtypes = [vp, vp, vp, vp] + [i32] * 4 + [vp]
             L.topk_attn_workspace_bytes.argtypes = [i32] * 8
             L.topk_attn_workspace_bytes.restype = sz
             L.topk_ffn_workspace_bytes.argtypes = [i32] * 4
@@ -56,7 +57,8 @@ def lib() -> ctypes.CDLL:
             L.topk_set_wait_limit_us.restype = ctypes.c_longlong
             L.topk_debug_skip_arrive.argtypes = [i32]
             for f in ("topk_attn_fwd", "topk_attn_fwd_indices", "topk_ffn_fwd", "topk_ffn_fwd_indices",
-                      "topk_attn_fwd_host", "topk_ffn_fwd_host", "topk_check", "topk_last_launch_count",
+                      "topk_attn_fwd_host", "topk_ffn_fwd_host", "topk_ffn_fwd_noalloc", "topk_check",
+                      "topk_last_launch_count",
                       "topk_debug_skip_arrive"):
                 getattr(L, f).restype = i32
             _lib = L
@@ -164,6 +166,22 @@ def topk_ffn_fwd_host(x, W1, W2, out, topk: int, stream=None) -> None:
     N, dm, dff = _ffn_dims(x, W1, W2, out)
     rc = lib().topk_ffn_fwd_host(_ptr(x), _ptr(W1), _ptr(W2), _ptr(out), N, dm, dff, int(topk), _stream(stream))
     _check(rc, "topk_ffn_fwd_host")
+
+
+# Size of the fixed scratch buffer of topk_ffn_fwd_noalloc (include/topk_attention.h).
+TOPK_FFN_NOALLOC_SCRATCH_BYTES = 32 << 20
+
+
+def topk_ffn_fwd_noalloc(x, W1, W2, out, topk: int, stream=None) -> None:
+    """topk_ffn_fwd for callers that cannot allocate device memory at call time.
+
+    Scratch comes from one fixed buffer inside the library instead of the
+    stream-ordered pool (see the C header for the size limit and why calls
+    that overlap on the GPU must be serialised).
+    """
+    N, dm, dff = _ffn_dims(x, W1, W2, out)
+    rc = lib().topk_ffn_fwd_noalloc(_ptr(x), _ptr(W1), _ptr(W2), _ptr(out), N, dm, dff, int(topk), _stream(stream))
+    _check(rc, "topk_ffn_fwd_noalloc")
 
 
 def topk_attn_workspace_bytes(B, H, Lq, Lk, d, topk, chunk, dtype) -> int:
