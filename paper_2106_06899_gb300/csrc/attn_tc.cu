@@ -33,15 +33,18 @@ constexpr int kThreads = 192;
 
 template <int D>
 struct TcShape;
+// N: keys per tile (MMA N); S: key-ring stages; OW: scores per selection call
 template <>
 struct TcShape<64> {
   static constexpr int N = 256;
   static constexpr int S = 2;
+  static constexpr int OW = 64;
 };
 template <>
 struct TcShape<128> {
   static constexpr int N = 64;
-  static constexpr int S = 3;
+  static constexpr int S = 2;
+  static constexpr int OW = 32;
 };
 
 using Sel = RowHeap<BM>;
@@ -61,10 +64,12 @@ struct Layout {
   static constexpr size_t kMaxSmem = 232448;
   static constexpr size_t kFixed = 1024 + OFF_SEL + CTRL_BYTES;
 
-  // pending score groups per row: as many as fit, at most 24 (0: the heap does not fit)
+  // pending score groups per row: as many as fit, at most 24; a selection call
+  // adds up to OW/8 groups, so fewer than OW/8 + 1 does not work (0)
+  static constexpr int kMinRec = TcShape<D>::OW / 8 + 1;
   static int rec_cap(int topk) {
     const size_t heap = static_cast<size_t>(topk) * BM * 8;
-    if (kFixed + heap + Sel::bytes(0, 4) >= kMaxSmem) return 0;
+    if (kFixed + heap + Sel::bytes(0, kMinRec) > kMaxSmem) return 0;
     const size_t room = (kMaxSmem - kFixed - heap) / (BM * 36);
     return room >= 24 ? 24 : static_cast<int>(room);
   }
@@ -299,7 +304,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           const uint32_t j0 = jt + static_cast<uint32_t>(c * 64);
           if (static_cast<int>(j0) + 64 > lim_min) mask_scores(vals, j0, lim);
-          heap.offer(vals, j0);
+          constexpr int OW = TcShape<D>::OW;
+#pragma unroll
+          for (int h = 0; h < 64 / OW; ++h)
+            heap.offer(reinterpret_cast<const float(&)[OW]>(vals[h * OW]), j0 + static_cast<uint32_t>(h * OW));
         }
       }
       if (!ok) break;
@@ -349,8 +357,8 @@ int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st
 
 bool attn_tc_supports(const AttnArgs& a) {
   if (a.dtype != 1 || a.topk > kTcMaxK) return false;
-  if (a.d == 64) return Layout<64>::rec_cap(a.topk) >= 4;
-  if (a.d == 128) return Layout<128>::rec_cap(a.topk) >= 4;
+  if (a.d == 64) return Layout<64>::rec_cap(a.topk) >= Layout<64>::kMinRec;
+  if (a.d == 128) return Layout<128>::rec_cap(a.topk) >= Layout<128>::kMinRec;
   return false;
 }
 

@@ -148,9 +148,8 @@ struct RowHeap {
   // Expand every lane's pending records into its heap, lanes in lockstep.
   // For each record slot every lane forms the mask of its elements that
   // still beat tau; then the warp pushes one element per lane per step, so
-  // that one push body serves all lanes at once.  Not inlined: it is the
-  // rare path of every unrolled offer8.
-  __device__ __noinline__ void flush() {
+  // that one push body serves all lanes at once.
+  __device__ __forceinline__ void flush() {
     const int mxr = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(rc));
     for (int i = 0; i < mxr; ++i) {
       unsigned msk = 0;
@@ -175,22 +174,31 @@ struct RowHeap {
     rc = 0;
   }
 
-  // Offer 8 scores with key indices j0 .. j0+7 (ascending).
-  __device__ __forceinline__ void offer8(const float* v, uint32_t j0) {
-    const float m = max3f(max3f(v[0], v[1], v[2]), max3f(v[3], v[4], v[5]), fmaxf(v[6], v[7]));
-    if (m > tau) {
-      rlo[rc * ROWS] = make_float4(v[0], v[1], v[2], v[3]);
-      rhi[rc * ROWS] = make_float4(v[4], v[5], v[6], v[7]);
-      rj[rc * ROWS] = j0;
-      ++rc;
-    }
-    if (__any_sync(0xffffffffu, rc == gr)) flush();
-  }
-
+  // Offer W scores with key indices j0 .. j0+W-1 (ascending).  The maxima of
+  // the W/8 groups are independent (computed first, for instruction-level
+  // parallelism); each group that beats tau becomes one record; one warp
+  // vote per call decides whether to flush, keeping every lane's record
+  // count at most gr - W/8 between calls.
   template <int W>
   __device__ __forceinline__ void offer(const float (&v)[W], uint32_t j0) {
+    constexpr int G = W / 8;
+    float m[G];
 #pragma unroll
-    for (int g = 0; g < W / 8; ++g) offer8(&v[8 * g], j0 + 8 * g);
+    for (int g = 0; g < G; ++g)
+      m[g] = max3f(max3f(v[8 * g], v[8 * g + 1], v[8 * g + 2]), max3f(v[8 * g + 3], v[8 * g + 4], v[8 * g + 5]),
+                   fmaxf(v[8 * g + 6], v[8 * g + 7]));
+    int r = rc;
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      if (m[g] > tau) {
+        rlo[r * ROWS] = make_float4(v[8 * g], v[8 * g + 1], v[8 * g + 2], v[8 * g + 3]);
+        rhi[r * ROWS] = make_float4(v[8 * g + 4], v[8 * g + 5], v[8 * g + 6], v[8 * g + 7]);
+        rj[r * ROWS] = j0 + 8 * g;
+        ++r;
+      }
+    }
+    rc = r;
+    if (__any_sync(0xffffffffu, rc > gr - G)) flush();
   }
 
   // After the last key: merge what is pending, then heap-sort in place so
