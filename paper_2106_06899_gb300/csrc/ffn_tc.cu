@@ -41,8 +41,10 @@ constexpr int NBINS = 64;
 constexpr uint32_t A_BYTES = BM * KC * 2;  // 16 KB
 constexpr uint32_t B_BYTES = NT * KC * 2;  // 32 KB
 constexpr uint32_t ST_BYTES = A_BYTES + B_BYTES;
+constexpr int GR = 10;    // pending score groups per row (a 64-score call adds up to 8)
 constexpr size_t OFF_HIST = static_cast<size_t>(S) * ST_BYTES;
-constexpr size_t OFF_CTRL = OFF_HIST + static_cast<size_t>(NBINS) * BM * 4;
+constexpr size_t OFF_REC = OFF_HIST + static_cast<size_t>(NBINS) * BM * 4;
+constexpr size_t OFF_CTRL = OFF_REC + static_cast<size_t>(GR) * BM * 36;
 constexpr size_t SMEM_A = 1024 + OFF_CTRL + 256;
 
 constexpr int kFinalThreads = 256;
@@ -164,6 +166,65 @@ struct RowCand {
         base += static_cast<float>(sh) * width;
       }
     }
+  }
+
+  // Pending score groups ([slot][row] records: 8 scores and the first key).
+  float4* rlo;
+  float4* rhi;
+  uint32_t* rj;
+  int rc;
+
+  // Expand every lane's records into its candidate list, lanes in lockstep:
+  // per record slot each lane forms the mask of its elements >= Lf, then the
+  // warp appends one element per lane per step.
+  __device__ __forceinline__ void flush(float Lf, bool active) {
+    const int mxr = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(active ? rc : 0));
+    for (int i = 0; i < mxr; ++i) {
+      unsigned msk = 0;
+      uint32_t j0 = 0;
+      if (active && i < rc) {
+        const float4 a = rlo[i * BM];
+        const float4 b = rhi[i * BM];
+        j0 = rj[i * BM];
+        msk = (a.x >= Lf ? 1u : 0u) | (a.y >= Lf ? 2u : 0u) | (a.z >= Lf ? 4u : 0u) | (a.w >= Lf ? 8u : 0u) |
+              (b.x >= Lf ? 16u : 0u) | (b.y >= Lf ? 32u : 0u) | (b.z >= Lf ? 64u : 0u) | (b.w >= Lf ? 128u : 0u);
+      }
+      while (__any_sync(0xffffffffu, msk != 0)) {
+        if (msk) {
+          const int e = __ffs(msk) - 1;
+          msk &= msk - 1;
+          const float v = e < 4 ? reinterpret_cast<const float*>(rlo + i * BM)[e]
+                                : reinterpret_cast<const float*>(rhi + i * BM)[e - 4];
+          add(v, j0 + e);
+        }
+      }
+    }
+    rc = 0;
+  }
+
+  // Offer 64 scores (key indices j0..j0+63) against the bound Lf: each group
+  // of 8 whose maximum reaches Lf becomes one record (NaN, used for keys past
+  // d_ff, never does).
+  __device__ __forceinline__ void offer64(const float (&v)[64], uint32_t j0, float Lf, bool active) {
+    float m[8];
+#pragma unroll
+    for (int g = 0; g < 8; ++g)
+      m[g] = max3f(max3f(v[8 * g], v[8 * g + 1], v[8 * g + 2]), max3f(v[8 * g + 3], v[8 * g + 4], v[8 * g + 5]),
+                   fmaxf(v[8 * g + 6], v[8 * g + 7]));
+    if (active) {
+      int r = rc;
+#pragma unroll
+      for (int g = 0; g < 8; ++g) {
+        if (m[g] >= Lf) {
+          rlo[r * BM] = make_float4(v[8 * g], v[8 * g + 1], v[8 * g + 2], v[8 * g + 3]);
+          rhi[r * BM] = make_float4(v[8 * g + 4], v[8 * g + 5], v[8 * g + 6], v[8 * g + 7]);
+          rj[r * BM] = j0 + 8 * g;
+          ++r;
+        }
+      }
+      rc = r;
+    }
+    if (__any_sync(0xffffffffu, active && rc > GR - 8)) flush(Lf, active);
   }
 };
 
@@ -306,6 +367,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     rc.hist = hist_mem + row;
     rc.k = topk;
     rc.cap = cap;
+    rc.rlo = reinterpret_cast<float4*>(smem + OFF_REC) + row;
+    rc.rhi = reinterpret_cast<float4*>(smem + OFF_REC + static_cast<size_t>(GR) * BM * 16) + row;
+    rc.rj = reinterpret_cast<uint32_t*>(smem + OFF_REC + static_cast<size_t>(GR) * BM * 32) + row;
+    rc.rc = 0;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
       int rt, sl, t0, t1;
       decode(u, rt, sl);
@@ -355,19 +420,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int e = 0; e < 64; ++e)
               if (j0 + e >= static_cast<uint32_t>(d_ff)) v[e] = __uint_as_float(0x7fc00000u);  // NaN: never kept
           }
-          if (row_ok && !rc.dead) {
-#pragma unroll
-            for (int g = 0; g < 8; ++g) {
-              const float* w = &v[8 * g];
-              const float m = max3f(max3f(w[0], w[1], w[2]), max3f(w[3], w[4], w[5]), fmaxf(w[6], w[7]));
-              if (m >= L) {
-#pragma unroll
-                for (int e = 0; e < 8; ++e)
-                  if (w[e] >= L) rc.add(w[e], j0 + 8 * g + e);
-              }
-            }
-          }
+          rc.offer64(v, j0, L, row_ok && !rc.dead);
         }
+        // the tile's pending groups go to the list before the bound moves
+        if (__any_sync(0xffffffffu, row_ok && !rc.dead && rc.rc > 0)) rc.flush(L, row_ok && !rc.dead);
         if (!row_ok || rc.dead) continue;
         rc.refresh();
         const uint32_t lkey = rc.L > -INFINITY ? ord_f32(rc.L) : 0u;
@@ -405,26 +461,47 @@ __global__ void __launch_bounds__(kThreads, 1)
 
 // One CTA per token row: exact top-k among its candidates, ReLU, W2 gather.
 //
-// Only candidates >= L (the row's shared bound) can be in the top-k.  If
-// more of them than fit in shared memory remain, an MSB-first radix pass
-// over the ordered score keys (8 bits at a time, counted in shared memory)
-// narrows the set: after each pass, every key whose leading bits exceed the
-// chosen prefix is certainly kept, and those equal to it are still open;
-// once kept + open fits, all of them are collected.  The exact top-k is
-// then a bitonic sort of the packed keys (score descending, index
-// ascending).
+// Only candidates >= L (the row's shared bound) can be in the top-k.  An
+// MSB-first radix select over their ordered score keys (11, 11 and 10 bits;
+// histograms in shared memory, increments aggregated per warp with
+// __match_any_sync so that equal digits do not serialise) finds the exact
+// k-th largest score t and how many keys equal to t are needed.  The kept
+// set is every key with score > t plus the needed keys equal to t with the
+// lowest indices (the tie rule); it is then sorted best first with a
+// bitonic sort of the packed keys.
+constexpr int kHistBins = 2048;
+
+__device__ __forceinline__ void warp_hist_add(uint32_t* hist, uint32_t d, bool valid) {
+  const unsigned peers = __match_any_sync(0xffffffffu, valid ? d : 0xFFFFFFFFu);
+  const int lane = threadIdx.x & 31;
+  if (valid && lane == __ffs(peers) - 1) atomicAdd(&hist[d], static_cast<unsigned>(__popc(peers)));
+}
+
+// Warp-aggregated append: returns this lane's slot (or -1 if !take).
+__device__ __forceinline__ int warp_append(int* counter, bool take) {
+  const unsigned bal = __ballot_sync(0xffffffffu, take);
+  if (!bal) return -1;
+  const int lane = threadIdx.x & 31;
+  int base = 0;
+  if (lane == __ffs(bal) - 1) base = atomicAdd(counter, __popc(bal));
+  base = __shfl_sync(0xffffffffu, base, __ffs(bal) - 1);
+  return take ? base + __popc(bal & ((1u << lane) - 1u)) : -1;
+}
+
 __global__ void __launch_bounds__(kFinalThreads)
     ffn_finalize_kernel(const __nv_bfloat16* __restrict__ W2, float* __restrict__ out, int d_model, int topk,
                         int n_sl, int cap, const uint2* __restrict__ cand, const int* __restrict__ cand_cnt,
                         const uint32_t* __restrict__ row_tau, int32_t* __restrict__ idx,
                         float* __restrict__ score, DevCtl ctl) {
-  extern __shared__ uint64_t keys[];  // [kFinalMaxCand]
-  __shared__ uint32_t hist[256];
-  __shared__ int n_keys, bad, sh_digit, sh_above;
+  extern __shared__ uint64_t keys[];  // [kFinalMaxCand]; the first kHistBins words double as the histogram
+  __shared__ uint32_t csum[kFinalThreads];
+  __shared__ int n_keys, n_ties, bad, sh_digit, sh_above;
+  uint32_t* hist = reinterpret_cast<uint32_t*>(keys);
   const int row = blockIdx.x;
   const int tid = threadIdx.x;
   if (tid == 0) {
     n_keys = 0;
+    n_ties = 0;
     bad = 0;
   }
   __syncthreads();
@@ -439,68 +516,126 @@ __global__ void __launch_bounds__(kFinalThreads)
     if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
     return;
   }
-  // visit every candidate of the row that is >= L: f(ord, index)
+  // visit every candidate slot of the row; all threads iterate together
   auto for_each = [&](auto&& f) {
     for (int sl = 0; sl < n_sl; ++sl) {
       const int c = cand_cnt[static_cast<size_t>(row) * n_sl + sl];
       const uint2* lst = cand + (static_cast<size_t>(row) * n_sl + sl) * cap;
-      for (int i = tid; i < c; i += kFinalThreads) {
-        const uint2 e = lst[i];
-        const float sc = __uint_as_float(e.x);
-        if (sc >= L) f(ord_f32(sc), e.y);
+      for (int b0 = 0; b0 < c; b0 += kFinalThreads) {
+        const int i = b0 + tid;
+        uint2 e = make_uint2(0u, 0u);
+        bool valid = i < c;
+        if (valid) {
+          e = lst[i];
+          valid = __uint_as_float(e.x) >= L;
+        }
+        f(valid, valid ? ord_f32(__uint_as_float(e.x)) : 0u, e.y);
       }
     }
   };
-  // radix narrowing: keys with (ord >> (32 - plen)) > prefix are kept for sure
-  uint32_t prefix = 0;
-  int plen = 0, remaining = topk, total = 0;
-  for (;;) {
-    if (tid < 256) hist[tid] = 0;
+  // radix select: the k-th largest ordered key among the candidates >= L
+  uint32_t prefix = 0, pmask = 0;
+  int remaining = topk;
+  const int shifts[3] = {21, 10, 0};
+  const uint32_t dmasks[3] = {0x7FFu, 0x7FFu, 0x3FFu};
+#pragma unroll
+  for (int pass = 0; pass < 3; ++pass) {
+    for (int i = tid; i < kHistBins; i += kFinalThreads) hist[i] = 0u;
     __syncthreads();
-    if (plen == 32) break;
-    const int shift = 24 - plen;
-    for_each([&](uint32_t o, uint32_t) {
-      if (plen == 0 || (o >> (32 - plen)) == prefix) atomicAdd(&hist[(o >> shift) & 255u], 1u);
+    const int sh = shifts[pass];
+    const uint32_t dm = dmasks[pass];
+    for_each([&](bool valid, uint32_t o, uint32_t) {
+      const bool mine = valid && (o & pmask) == prefix;
+      warp_hist_add(hist, (o >> sh) & dm, mine);
     });
+    __syncthreads();
+    // chunk sums from the top bin down, then one thread locates the digit
+    const int nb = static_cast<int>(dm) + 1, per = (nb + kFinalThreads - 1) / kFinalThreads;
+    uint32_t cs = 0;
+    for (int q = 0; q < per; ++q) {
+      const int bin = nb - 1 - (tid * per + q);
+      if (bin >= 0) cs += hist[bin];
+    }
+    csum[tid] = cs;
     __syncthreads();
     if (tid == 0) {
       uint32_t cum = 0;
-      int d = 255;
-      for (; d > 0; --d) {
-        if (cum + hist[d] >= static_cast<uint32_t>(remaining)) break;
-        cum += hist[d];
+      int t = 0;
+      for (; t < kFinalThreads; ++t) {
+        if (cum + csum[t] >= static_cast<uint32_t>(remaining)) break;
+        cum += csum[t];
       }
-      sh_digit = d;
+      int digit = -1;
+      for (int q = 0; q < per && t < kFinalThreads; ++q) {
+        const int bin = nb - 1 - (t * per + q);
+        if (bin < 0) break;
+        if (cum + hist[bin] >= static_cast<uint32_t>(remaining)) {
+          digit = bin;
+          break;
+        }
+        cum += hist[bin];
+      }
+      sh_digit = digit;
       sh_above = static_cast<int>(cum);
     }
     __syncthreads();
-    const int d = sh_digit;
-    const int above = sh_above;
-    const int open = static_cast<int>(hist[d]);
-    prefix = (prefix << 8) | static_cast<uint32_t>(d);
-    plen += 8;
-    remaining -= above;
-    total = (topk - remaining) + open;
-    __syncthreads();
-    if (total <= kFinalMaxCand) break;
-  }
-  if (total > kFinalMaxCand) {  // more exact ties than shared memory holds
-    if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
-    return;
-  }
-  for_each([&](uint32_t o, uint32_t j) {
-    if (plen == 0 || (o >> (32 - plen)) >= prefix) {
-      const int pos = atomicAdd(&n_keys, 1);
-      if (pos < kFinalMaxCand) keys[pos] = (static_cast<uint64_t>(o) << 32) | static_cast<uint64_t>(~j);
+    if (sh_digit < 0) {  // fewer candidates than k: cannot happen unless the lists are inconsistent
+      if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
+      return;
     }
+    prefix |= static_cast<uint32_t>(sh_digit) << sh;
+    pmask |= dm << sh;
+    remaining -= sh_above;
+    __syncthreads();
+  }
+  // prefix = ordered key of the k-th largest score; `remaining` keys equal to it are kept
+  const uint32_t thr = prefix;
+  uint32_t* ties = reinterpret_cast<uint32_t*>(keys + topk);  // indices of keys equal to thr
+  const int tie_cap = (kFinalMaxCand - topk) * 2;
+  for_each([&](bool valid, uint32_t o, uint32_t j) {
+    const int pa = warp_append(&n_keys, valid && o > thr);
+    if (pa >= 0 && pa < topk) keys[pa] = (static_cast<uint64_t>(o) << 32) | static_cast<uint64_t>(~j);
+    const int pt = warp_append(&n_ties, valid && o == thr);
+    if (pt >= 0 && pt < tie_cap) ties[pt] = j;
   });
   __syncthreads();
-  const int n = n_keys;
-  if (n > kFinalMaxCand || n < topk) {
+  const int na = n_keys, nt = n_ties;
+  if (na + remaining != topk || nt < remaining || nt > tie_cap) {
     if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
     return;
   }
-  // bitonic sort, descending, over the next power of two (padding keys rank last)
+  // the `remaining` lowest indices among the ties (ascending bitonic sort of the tie indices)
+  if (nt > remaining) {
+    int m = 1;
+    while (m < nt) m <<= 1;
+    if (m > tie_cap) {
+      if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
+      return;
+    }
+    for (int i = nt + tid; i < m; i += kFinalThreads) ties[i] = 0xFFFFFFFFu;
+    __syncthreads();
+    for (int size = 2; size <= m; size <<= 1) {
+      for (int stride = size >> 1; stride > 0; stride >>= 1) {
+        for (int i = tid; i < (m >> 1); i += kFinalThreads) {
+          const int lo = 2 * i - (i & (stride - 1));
+          const int hi = lo + stride;
+          const bool asc = (lo & size) == 0;
+          const uint32_t x = ties[lo], y = ties[hi];
+          if ((x > y) == asc) {
+            ties[lo] = y;
+            ties[hi] = x;
+          }
+        }
+        __syncthreads();
+      }
+    }
+  }
+  __syncthreads();
+  for (int t = tid; t < remaining; t += kFinalThreads)
+    keys[na + t] = (static_cast<uint64_t>(thr) << 32) | static_cast<uint64_t>(~ties[t]);
+  __syncthreads();
+  const int n = topk;
+  // bitonic sort of the k kept keys, descending (padding keys rank last)
   int m = 1;
   while (m < n) m <<= 1;
   for (int i = n + tid; i < m; i += kFinalThreads) keys[i] = 0ull;

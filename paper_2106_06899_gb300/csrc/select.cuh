@@ -123,52 +123,58 @@ struct RowHeap {
     put(p, x);
   }
 
+  // Add x: while the heap is not full it is appended (the heap is built
+  // once, when the k-th entry arrives); afterwards it replaces the root if it
+  // ranks above it.
   __device__ __forceinline__ void push(uint64_t x) {
     if (n < k) {
-      int c = n;
-      while (c > 0) {
-        const int p = (c - 1) >> 2;
-        const uint64_t pk = get(p);
-        if (pk <= x) break;
-        put(c, pk);
-        c = p;
-      }
-      put(c, x);
+      put(n, x);
       if (++n == k) {
+        for (int p = (k - 2) / 4; p >= 0; --p) sift_down(get(p), p, k);
         root = get(0);
         tau = key_score(root);
       }
     } else if (x > root) {
-      sift_down(x, 0, n);
+      sift_down(x, 0, k);
       root = get(0);
       tau = key_score(root);
     }
   }
 
-  // Expand every lane's pending records into its heap, lanes in lockstep.
-  // For each record slot every lane forms the mask of its elements that
-  // still beat tau; then the warp pushes one element per lane per step, so
-  // that one push body serves all lanes at once.
+  // Expand every lane's pending records into its heap.  Each lane walks its
+  // own records in order (ascending key index) and offers one element per
+  // step; the warp steps together until every lane is done, so one push body
+  // serves all lanes at once and no lane waits on another lane's record
+  // slot.  Elements are re-checked against the current tau.
   __device__ __forceinline__ void flush() {
-    const int mxr = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(rc));
-    for (int i = 0; i < mxr; ++i) {
-      unsigned msk = 0;
-      uint32_t j0 = 0;
-      const float* sc = reinterpret_cast<const float*>(rlo + i * ROWS);  // scores 0..3, then 4..7 in rhi
-      if (i < rc) {
+    int i = 0;
+    unsigned msk = 0;
+    uint32_t j0 = 0;
+    float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f, v4 = 0.f, v5 = 0.f, v6 = 0.f, v7 = 0.f;
+    auto next_record = [&]() {
+      while (msk == 0 && i < rc) {
         const float4 a = rlo[i * ROWS];
         const float4 b = rhi[i * ROWS];
         j0 = rj[i * ROWS];
-        msk = (a.x > tau ? 1u : 0u) | (a.y > tau ? 2u : 0u) | (a.z > tau ? 4u : 0u) | (a.w > tau ? 8u : 0u) |
-              (b.x > tau ? 16u : 0u) | (b.y > tau ? 32u : 0u) | (b.z > tau ? 64u : 0u) | (b.w > tau ? 128u : 0u);
+        v0 = a.x; v1 = a.y; v2 = a.z; v3 = a.w;
+        v4 = b.x; v5 = b.y; v6 = b.z; v7 = b.w;
+        msk = (v0 > tau ? 1u : 0u) | (v1 > tau ? 2u : 0u) | (v2 > tau ? 4u : 0u) | (v3 > tau ? 8u : 0u) |
+              (v4 > tau ? 16u : 0u) | (v5 > tau ? 32u : 0u) | (v6 > tau ? 64u : 0u) | (v7 > tau ? 128u : 0u);
+        ++i;
       }
-      while (__any_sync(0xffffffffu, msk != 0)) {
-        if (msk) {
-          const int e = __ffs(msk) - 1;
-          msk &= msk - 1;
-          const float v = e < 4 ? sc[e] : reinterpret_cast<const float*>(rhi + i * ROWS)[e - 4];
-          if (v > tau) push(make_key(v, j0 + e));
-        }
+    };
+    next_record();
+    while (__any_sync(0xffffffffu, msk != 0)) {
+      if (msk) {
+        const int e = __ffs(msk) - 1;
+        msk &= msk - 1;
+        // v[e] by bit-select (no dynamically indexed register array)
+        const float x01 = (e & 1) ? v1 : v0, x23 = (e & 1) ? v3 : v2;
+        const float x45 = (e & 1) ? v5 : v4, x67 = (e & 1) ? v7 : v6;
+        const float x03 = (e & 2) ? x23 : x01, x47 = (e & 2) ? x67 : x45;
+        const float x = (e & 4) ? x47 : x03;
+        if (x > tau) push(make_key(x, j0 + static_cast<uint32_t>(e)));
+        if (msk == 0) next_record();
       }
     }
     rc = 0;
@@ -203,8 +209,12 @@ struct RowHeap {
 
   // After the last key: merge what is pending, then heap-sort in place so
   // that slots 0 .. n-1 hold the kept keys in selection order (best first).
+  // A row that never filled its heap (fewer than k valid keys) is heapified
+  // first: its entries were appended unordered.
   __device__ __forceinline__ void finish() {
     flush();
+    if (n < k && n > 1)
+      for (int p = (n - 2) / 4; p >= 0; --p) sift_down(get(p), p, n);
     for (int m = n - 1; m > 0; --m) {
       const uint64_t x = get(m);
       put(m, get(0));
