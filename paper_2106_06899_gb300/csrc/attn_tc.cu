@@ -70,7 +70,7 @@ struct Layout {
   static int rec_cap(int topk) {
     const size_t heap = static_cast<size_t>(topk) * BM * 8;
     if (kFixed + heap + Sel::bytes(0, kMinRec) > kMaxSmem) return 0;
-    const size_t room = (kMaxSmem - kFixed - heap) / (BM * 36);
+    const size_t room = (kMaxSmem - kFixed - heap) / (BM * 44);
     return room >= 24 ? 24 : static_cast<int>(room);
   }
   __host__ __device__ static size_t sel_bytes(int topk, int gr) { return (Sel::bytes(topk, gr) + 15) & ~size_t(15); }

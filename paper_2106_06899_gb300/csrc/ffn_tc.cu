@@ -60,10 +60,14 @@ Plan make_plan(int N, int d_model, int d_ff, int topk, int num_sms) {
   Plan p{};
   p.n_rt = (N + BM - 1) / BM;
   p.tiles = (d_ff + NT - 1) / NT;
-  // slices: minimise waves x tiles-per-slice, plus a small charge per slice
-  // (each slice has its own warm-up of k candidates)
+  // slices: minimise waves x tiles-per-slice, plus a small charge per slice.
+  // Each slice bounds only its own k-th score, so a slice keeps about
+  // k (1 + ln(slice/k)) candidates per row: slices are kept at >= 32 k keys
+  // (unless that leaves fewer units than SMs / 4) to hold that volume down.
   double best = 1e30;
-  const int max_sl = std::max(1, std::min(p.tiles, 64));
+  int max_sl = std::max(1, std::min(p.tiles, 64));
+  const int by_k = std::max(1, d_ff / (32 * std::max(topk, 1)));
+  if (by_k < max_sl && static_cast<long>(p.n_rt) * by_k * 4 >= num_sms) max_sl = by_k;
   for (int sl = 1; sl <= max_sl; ++sl) {
     const long units = static_cast<long>(p.n_rt) * sl;
     const long waves = (units + num_sms - 1) / num_sms;
@@ -76,7 +80,9 @@ Plan make_plan(int N, int d_model, int d_ff, int topk, int num_sms) {
   }
   p.n_units = p.n_rt * p.n_sl;
   const int slice_keys = ((p.tiles + p.n_sl - 1) / p.n_sl) * NT;
-  const int want = 4 * topk + 1024;
+  // room for about k (1 + ln(slice/k)) candidates plus the bound's lag,
+  // so that the in-place compaction (a slow path) stays rare
+  const int want = 6 * topk + 1024;
   p.cap = ((std::min(slice_keys, want) + 63) / 64) * 64;
   const size_t rows_sl = static_cast<size_t>(N) * p.n_sl;
   p.off_cnt = rows_sl * p.cap * sizeof(uint2);
@@ -536,6 +542,7 @@ __global__ void __launch_bounds__(kFinalThreads)
   // radix select: the k-th largest ordered key among the candidates >= L
   uint32_t prefix = 0, pmask = 0;
   int remaining = topk;
+  bool direct = false;
   const int shifts[3] = {21, 10, 0};
   const uint32_t dmasks[3] = {0x7FFu, 0x7FFu, 0x3FFu};
 #pragma unroll
@@ -586,8 +593,45 @@ __global__ void __launch_bounds__(kFinalThreads)
     prefix |= static_cast<uint32_t>(sh_digit) << sh;
     pmask |= dm << sh;
     remaining -= sh_above;
+    const int kept_or_open = (topk - remaining) + static_cast<int>(hist[sh_digit]);
     __syncthreads();
+    if (pass == 0 && kept_or_open <= kFinalMaxCand) {
+      // everything at or above the k-th key's leading 11 bits fits in shared
+      // memory: collect it and finish there (one more read of the lists)
+      for_each([&](bool valid, uint32_t o, uint32_t j) {
+        const int pa = warp_append(&n_keys, valid && (o & pmask) >= prefix);
+        if (pa >= 0 && pa < kFinalMaxCand) keys[pa] = (static_cast<uint64_t>(o) << 32) | static_cast<uint64_t>(~j);
+      });
+      __syncthreads();
+      const int nc = n_keys;
+      if (nc != kept_or_open || nc < topk) {
+        if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
+        return;
+      }
+      int m2 = 1;
+      while (m2 < nc) m2 <<= 1;
+      for (int i = nc + tid; i < m2; i += kFinalThreads) keys[i] = 0ull;
+      __syncthreads();
+      for (int size = 2; size <= m2; size <<= 1) {
+        for (int stride = size >> 1; stride > 0; stride >>= 1) {
+          for (int i = tid; i < (m2 >> 1); i += kFinalThreads) {
+            const int lo = 2 * i - (i & (stride - 1));
+            const int hi = lo + stride;
+            const bool desc = (lo & size) == 0;
+            const uint64_t a = keys[lo], b = keys[hi];
+            if ((a < b) == desc) {
+              keys[lo] = b;
+              keys[hi] = a;
+            }
+          }
+          __syncthreads();
+        }
+      }
+      direct = true;  // keys[0 .. topk) are the kept keys, best first
+      break;
+    }
   }
+  if (!direct) {
   // prefix = ordered key of the k-th largest score; `remaining` keys equal to it are kept
   const uint32_t thr = prefix;
   uint32_t* ties = reinterpret_cast<uint32_t*>(keys + topk);  // indices of keys equal to thr
@@ -654,6 +698,7 @@ __global__ void __launch_bounds__(kFinalThreads)
       }
       __syncthreads();
     }
+  }
   }
   // ReLU over the kept scores and the weighted sum of W2 rows (fp32), eight
   // rows in flight per thread

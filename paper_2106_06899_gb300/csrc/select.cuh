@@ -63,6 +63,7 @@ struct RowHeap {
   float4* rlo;     // &records_lo[0][this row]: scores 0..3
   float4* rhi;     // &records_hi[0][this row]: scores 4..7
   uint32_t* rj;    // &records_j0[0][this row]
+  uint8_t* stage;  // &stage[0][this row]: codes (record slot * 8 + element) of elements to offer
   int k;           // capacity
   int n;           // entries filled
   int rc;          // records pending
@@ -70,9 +71,10 @@ struct RowHeap {
   uint64_t root;   // heap[0] once full
   float tau;       // score of heap[0] once full, else -inf
 
-  // shared memory: heap k x ROWS x 8 bytes, then records gr x ROWS x 36 bytes
+  // shared memory: heap k x ROWS x 8 bytes, records gr x ROWS x 36 bytes,
+  // stage 8 gr x ROWS bytes (gr <= 32, so that a code fits in one byte)
   __host__ __device__ static constexpr size_t bytes(int k_, int gr_) {
-    return static_cast<size_t>(ROWS) * (static_cast<size_t>(k_) * 8 + static_cast<size_t>(gr_) * 36);
+    return static_cast<size_t>(ROWS) * (static_cast<size_t>(k_) * 8 + static_cast<size_t>(gr_) * 44);
   }
 
   __device__ __forceinline__ void init(uint8_t* smem, int row, int cap, int rec_cap) {
@@ -81,6 +83,7 @@ struct RowHeap {
     rlo = reinterpret_cast<float4*>(r) + row;
     rhi = reinterpret_cast<float4*>(r + static_cast<size_t>(rec_cap) * ROWS * 16) + row;
     rj = reinterpret_cast<uint32_t*>(r + static_cast<size_t>(rec_cap) * ROWS * 32) + row;
+    stage = r + static_cast<size_t>(rec_cap) * ROWS * 36 + row;
     k = cap;
     gr = rec_cap;
     n = 0;
@@ -141,40 +144,34 @@ struct RowHeap {
     }
   }
 
-  // Expand every lane's pending records into its heap.  Each lane walks its
-  // own records in order (ascending key index) and offers one element per
-  // step; the warp steps together until every lane is done, so one push body
-  // serves all lanes at once and no lane waits on another lane's record
-  // slot.  Elements are re-checked against the current tau.
+  // Expand every lane's pending records into its heap, in two phases.
+  // 1. Each lane lists, in key order, the elements of its own records that
+  //    beat tau (one-byte codes: record slot * 8 + element); predicated
+  //    stores, no cross-lane traffic.
+  // 2. The warp walks the lists in lockstep, one element per lane per step,
+  //    re-checking each against the current root: one heap replace body
+  //    serves all lanes at once.
   __device__ __forceinline__ void flush() {
-    int i = 0;
-    unsigned msk = 0;
-    uint32_t j0 = 0;
-    float v0 = 0.f, v1 = 0.f, v2 = 0.f, v3 = 0.f, v4 = 0.f, v5 = 0.f, v6 = 0.f, v7 = 0.f;
-    auto next_record = [&]() {
-      while (msk == 0 && i < rc) {
-        const float4 a = rlo[i * ROWS];
-        const float4 b = rhi[i * ROWS];
-        j0 = rj[i * ROWS];
-        v0 = a.x; v1 = a.y; v2 = a.z; v3 = a.w;
-        v4 = b.x; v5 = b.y; v6 = b.z; v7 = b.w;
-        msk = (v0 > tau ? 1u : 0u) | (v1 > tau ? 2u : 0u) | (v2 > tau ? 4u : 0u) | (v3 > tau ? 8u : 0u) |
-              (v4 > tau ? 16u : 0u) | (v5 > tau ? 32u : 0u) | (v6 > tau ? 64u : 0u) | (v7 > tau ? 128u : 0u);
-        ++i;
+    int cnt = 0;
+    for (int i = 0; i < rc; ++i) {
+      const float4 a = rlo[i * ROWS];
+      const float4 b = rhi[i * ROWS];
+      const float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        if (v[e] > tau) {
+          stage[cnt * ROWS] = static_cast<uint8_t>(i * 8 + e);
+          ++cnt;
+        }
       }
-    };
-    next_record();
-    while (__any_sync(0xffffffffu, msk != 0)) {
-      if (msk) {
-        const int e = __ffs(msk) - 1;
-        msk &= msk - 1;
-        // v[e] by bit-select (no dynamically indexed register array)
-        const float x01 = (e & 1) ? v1 : v0, x23 = (e & 1) ? v3 : v2;
-        const float x45 = (e & 1) ? v5 : v4, x67 = (e & 1) ? v7 : v6;
-        const float x03 = (e & 2) ? x23 : x01, x47 = (e & 2) ? x67 : x45;
-        const float x = (e & 4) ? x47 : x03;
-        if (x > tau) push(make_key(x, j0 + static_cast<uint32_t>(e)));
-        if (msk == 0) next_record();
+    }
+    const int mx = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(cnt));
+    for (int t = 0; t < mx; ++t) {
+      if (t < cnt) {
+        const int code = stage[t * ROWS];
+        const int i = code >> 3, e = code & 7;
+        const float x = reinterpret_cast<const float*>((e < 4 ? rlo : rhi) + i * ROWS)[e & 3];
+        if (x > tau) push(make_key(x, rj[i * ROWS] + static_cast<uint32_t>(e)));
       }
     }
     rc = 0;
