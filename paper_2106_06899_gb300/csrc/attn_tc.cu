@@ -47,10 +47,11 @@ struct TcShape<128> {
   static constexpr int OW = 32;
 };
 
-using Sel = RowHeap<BM>;
 
-template <int D>
+
+template <int D, int FK>
 struct Layout {
+  using Sel = RowHeap<BM, FK>;
   static constexpr int N = TcShape<D>::N;
   static constexpr int S = TcShape<D>::S;
   static constexpr int R = D / 64;  // 128-byte column blocks per row
@@ -68,8 +69,8 @@ struct Layout {
   // adds up to OW/8 groups, so fewer than OW/8 + 1 does not work (0)
   static constexpr int kMinRec = TcShape<D>::OW / 8 + 1;
   static int rec_cap(int topk) {
-    const size_t heap = static_cast<size_t>(topk) * BM * 8;
-    if (kFixed + heap + Sel::bytes(0, kMinRec) > kMaxSmem) return 0;
+    const size_t heap = Sel::bytes(topk, 0);
+    if (kFixed + Sel::bytes(topk, kMinRec) > kMaxSmem) return 0;
     const size_t room = (kMaxSmem - kFixed - heap) / (BM * 44);
     return room >= 24 ? 24 : static_cast<int>(room);
   }
@@ -99,13 +100,14 @@ __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, const
   }
 }
 
-template <int D>
+template <int D, int FK>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmk,
                    const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ out, int BH, int Lq, int Lk,
                    int topk, int rec_cap, int causal, int n_units, int32_t* __restrict__ idx,
                    float* __restrict__ score, DevCtl ctl) {
-  using L = Layout<D>;
+  using L = Layout<D, FK>;
+  using Sel = typename L::Sel;
   constexpr int N = L::N, S = L::S, R = L::R;
   constexpr uint32_t IDESC = idesc_bf16_f32(BM, N);
   constexpr uint32_t TMEM_COLS = 2 * N;
@@ -330,9 +332,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int D>
-int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
-  using L = Layout<D>;
+template <int D, int FK>
+int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
+  using L = Layout<D, FK>;
   const int BH = a.B * a.H;
   CUtensorMap tmq, tmk;
   if (!make_tmap_bf16_3d(&tmq, a.q, D, a.Lq, BH, BM)) return -1;
@@ -342,7 +344,7 @@ int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st
   // all TMEM columns it needs for its whole (persistent) lifetime.
   const size_t need = L::bytes(a.topk);
   const size_t smem = need > 120 * 1024 ? need : 120 * 1024;
-  auto kern = attn_tc_kernel<D>;
+  auto kern = attn_tc_kernel<D, FK>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
       cudaSuccess)
     return -1;
@@ -353,12 +355,19 @@ int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
+template <int D>
+int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
+  if (a.topk == 64 && Layout<D, 64>::rec_cap(64) >= Layout<D, 64>::kMinRec)
+    return launch_tc_k<D, 64>(a, ctl, num_sms, st);
+  return launch_tc_k<D, 0>(a, ctl, num_sms, st);
+}
+
 }  // namespace
 
 bool attn_tc_supports(const AttnArgs& a) {
   if (a.dtype != 1 || a.topk > kTcMaxK) return false;
-  if (a.d == 64) return Layout<64>::rec_cap(a.topk) >= Layout<64>::kMinRec;
-  if (a.d == 128) return Layout<128>::rec_cap(a.topk) >= Layout<128>::kMinRec;
+  if (a.d == 64) return Layout<64, 0>::rec_cap(a.topk) >= Layout<64, 0>::kMinRec;
+  if (a.d == 128) return Layout<128, 0>::rec_cap(a.topk) >= Layout<128, 0>::kMinRec;
   return false;
 }
 

@@ -57,8 +57,12 @@ __device__ __forceinline__ uint32_t key_index(uint64_t key) { return ~static_cas
 // memory round trips of a replace (log4 k levels of four independent loads).
 // ROWS = number of rows sharing the [slot][row] arrays (the row stride);
 // every call of offer*/flush/finish must be made by all 32 lanes of a warp.
-template <int ROWS>
+template <int ROWS, int FIXED_K = 0>
 struct RowHeap {
+  // FIXED_K == 64: an 8-ary heap of exactly 64 keys, padded with 9 sentinel
+  // slots (largest key) so that every interior node has 8 children: a root
+  // replacement is two fully unrolled levels of 8 independent loads.
+  static constexpr int kPad = FIXED_K == 64 ? 9 : 0;
   uint64_t* base;  // &heap[slot 0][this row]
   float4* rlo;     // &records_lo[0][this row]: scores 0..3
   float4* rhi;     // &records_hi[0][this row]: scores 4..7
@@ -71,15 +75,16 @@ struct RowHeap {
   uint64_t root;   // heap[0] once full
   float tau;       // score of heap[0] once full, else -inf
 
-  // shared memory: heap k x ROWS x 8 bytes, records gr x ROWS x 36 bytes,
-  // stage 8 gr x ROWS bytes (gr <= 32, so that a code fits in one byte)
+  // shared memory: heap (k + kPad) x ROWS x 8 bytes, records gr x ROWS x 36
+  // bytes, stage 8 gr x ROWS bytes (gr <= 32, so that a code fits in a byte)
   __host__ __device__ static constexpr size_t bytes(int k_, int gr_) {
-    return static_cast<size_t>(ROWS) * (static_cast<size_t>(k_) * 8 + static_cast<size_t>(gr_) * 44);
+    return static_cast<size_t>(ROWS) * (static_cast<size_t>(k_ + kPad) * 8 + static_cast<size_t>(gr_) * 44);
   }
 
   __device__ __forceinline__ void init(uint8_t* smem, int row, int cap, int rec_cap) {
     base = reinterpret_cast<uint64_t*>(smem) + row;
-    uint8_t* r = smem + static_cast<size_t>(cap) * ROWS * 8;
+    uint8_t* r = smem + static_cast<size_t>(cap + kPad) * ROWS * 8;
+    for (int q = 0; q < kPad; ++q) base[(cap + q) * ROWS] = ~0ull;  // sentinels never leave the leaves
     rlo = reinterpret_cast<float4*>(r) + row;
     rhi = reinterpret_cast<float4*>(r + static_cast<size_t>(rec_cap) * ROWS * 16) + row;
     rj = reinterpret_cast<uint32_t*>(r + static_cast<size_t>(rec_cap) * ROWS * 32) + row;
@@ -126,6 +131,42 @@ struct RowHeap {
     put(p, x);
   }
 
+  // 8-ary heap of 64 keys: children of node p are 8p+1 .. 8p+8; slots 64..72
+  // hold sentinels.  Replace the root by x and restore the heap order.
+  __device__ __forceinline__ void replace_root64(uint64_t x) {
+    int p = 0;
+    bool done = false;
+#pragma unroll
+    for (int level = 0; level < 2; ++level) {
+      const int c = 8 * p + 1;
+      uint64_t ch[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) ch[q] = get(c + q);
+      // argmin over 8 keys, tree of depth 3
+      uint64_t m2[4];
+      int i2[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const bool lo = ch[2 * q] <= ch[2 * q + 1];
+        m2[q] = lo ? ch[2 * q] : ch[2 * q + 1];
+        i2[q] = lo ? 2 * q : 2 * q + 1;
+      }
+      const bool l01 = m2[0] <= m2[1], l23 = m2[2] <= m2[3];
+      const uint64_t m01 = l01 ? m2[0] : m2[1], m23 = l23 ? m2[2] : m2[3];
+      const int i01 = l01 ? i2[0] : i2[1], i23 = l23 ? i2[2] : i2[3];
+      const bool lf = m01 <= m23;
+      const uint64_t a = lf ? m01 : m23;
+      const int ca = c + (lf ? i01 : i23);
+      if (!done && a < x) {
+        put(p, a);
+        p = ca;
+      } else {
+        done = true;
+      }
+    }
+    put(p, x);
+  }
+
   // Add x: while the heap is not full it is appended (the heap is built
   // once, when the k-th entry arrives); afterwards it replaces the root if it
   // ranks above it.
@@ -133,15 +174,47 @@ struct RowHeap {
     if (n < k) {
       put(n, x);
       if (++n == k) {
-        for (int p = (k - 2) / 4; p >= 0; --p) sift_down(get(p), p, k);
+        if constexpr (FIXED_K == 64) {
+          // build the 8-ary heap: nodes 8..1 (level 1), then the root
+          for (int p = 8; p >= 1; --p) sift_down8(get(p), p);
+          sift_down8(get(0), 0);
+        } else {
+          for (int p = (k - 2) / 4; p >= 0; --p) sift_down(get(p), p, k);
+        }
         root = get(0);
         tau = key_score(root);
       }
     } else if (x > root) {
-      sift_down(x, 0, k);
+      if constexpr (FIXED_K == 64) {
+        replace_root64(x);
+      } else {
+        sift_down(x, 0, k);
+      }
       root = get(0);
       tau = key_score(root);
     }
+  }
+
+  // Sift down in the 8-ary heap of 64 (used to build it and to sort it).
+  // m: number of live entries (slots >= m are treated as absent).
+  __device__ __forceinline__ void sift_down8(uint64_t x, int p, int m = 64) {
+    for (;;) {
+      const int c = 8 * p + 1;
+      if (c >= m) break;
+      uint64_t a = get(c);
+      int ca = c;
+      for (int q = c + 1; q < c + 8 && q < m; ++q) {
+        const uint64_t b = get(q);
+        if (b < a) {
+          a = b;
+          ca = q;
+        }
+      }
+      if (a >= x) break;
+      put(p, a);
+      p = ca;
+    }
+    put(p, x);
   }
 
   // Expand every lane's pending records into its heap, in two phases.
@@ -210,12 +283,22 @@ struct RowHeap {
   // first: its entries were appended unordered.
   __device__ __forceinline__ void finish() {
     flush();
-    if (n < k && n > 1)
-      for (int p = (n - 2) / 4; p >= 0; --p) sift_down(get(p), p, n);
-    for (int m = n - 1; m > 0; --m) {
-      const uint64_t x = get(m);
-      put(m, get(0));
-      sift_down(x, 0, m);
+    if constexpr (FIXED_K == 64) {
+      if (n < k && n > 1)
+        for (int p = (n - 2) / 8; p >= 0; --p) sift_down8(get(p), p, n);
+      for (int m = n - 1; m > 0; --m) {
+        const uint64_t x = get(m);
+        put(m, get(0));
+        sift_down8(x, 0, m);
+      }
+    } else {
+      if (n < k && n > 1)
+        for (int p = (n - 2) / 4; p >= 0; --p) sift_down(get(p), p, n);
+      for (int m = n - 1; m > 0; --m) {
+        const uint64_t x = get(m);
+        put(m, get(0));
+        sift_down(x, 0, m);
+      }
     }
   }
 };
