@@ -38,7 +38,7 @@ template <>
 struct TcShape<64> {
   static constexpr int N = 256;
   static constexpr int S = 2;
-  static constexpr int OW = 64;
+  static constexpr int OW = 32;
 };
 template <>
 struct TcShape<128> {

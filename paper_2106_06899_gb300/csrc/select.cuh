@@ -239,13 +239,23 @@ struct RowHeap {
       }
     }
     const int mx = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(cnt));
+    // software-pipelined: the next element's loads are issued before this push
+    auto fetch = [&](int t, float& x, uint32_t& j) {
+      const int code = stage[t * ROWS];
+      const int i = code >> 3, e = code & 7;
+      x = reinterpret_cast<const float*>((e < 4 ? rlo : rhi) + i * ROWS)[e & 3];
+      j = rj[i * ROWS] + static_cast<uint32_t>(e);
+    };
+    float x = -INFINITY;
+    uint32_t j = 0;
+    if (cnt > 0) fetch(0, x, j);
     for (int t = 0; t < mx; ++t) {
-      if (t < cnt) {
-        const int code = stage[t * ROWS];
-        const int i = code >> 3, e = code & 7;
-        const float x = reinterpret_cast<const float*>((e < 4 ? rlo : rhi) + i * ROWS)[e & 3];
-        if (x > tau) push(make_key(x, rj[i * ROWS] + static_cast<uint32_t>(e)));
-      }
+      float xn = -INFINITY;
+      uint32_t jn = 0;
+      if (t + 1 < cnt) fetch(t + 1, xn, jn);
+      if (t < cnt && x > tau) push(make_key(x, j));
+      x = xn;
+      j = jn;
     }
     rc = 0;
   }
@@ -348,7 +358,7 @@ __device__ __forceinline__ void softmax_gather_store(const Sel& h, const T* __re
 #pragma unroll
     for (int c = 0; c < SL; ++c) acc[c] = 0.0f;
     float z = 0.0f;
-#pragma unroll 1
+#pragma unroll 2
     for (int t = 0; t < n; ++t) {
       const uint64_t key = h.get(t);
       const float w = expf(key_score(key) - m);
