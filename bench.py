@@ -42,6 +42,7 @@ def parse_args():
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="long_65k")
     p.add_argument("--L", type=int, default=0, help="override Lq = Lk (profiling on a small case)")
+    p.add_argument("--ffn-tokens", type=int, default=0, help="override the FF token count N (profiling)")
     p.add_argument("--e2e-steps", type=int, default=3)
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU work budget of the oracle baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -99,6 +100,8 @@ def workload(args):
     w = W.WORKLOADS[args.workload]
     if args.L:
         w = w.with_(Lq=args.L, Lk=args.L) if w.kind == "attn" else w.with_(d_ff=args.L)
+    if args.ffn_tokens and w.kind == "ffn":
+        w = w.with_(N=args.ffn_tokens)
     return w
 
 
@@ -237,6 +240,25 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+# ------------------------------------------------------------------ replicas
+def replica_throughput(ms_local: float, tokens_per_rank: int, device: str = "cuda"):
+    """Whole-job throughput of independent replicas, one per rank.
+
+    The path has no exchange step, so ranks run the same workload on their own GPU with no
+    collective on the data path; the job's rate is every rank's tokens over the SLOWEST rank's
+    time (MAX over ranks, the only collective, used for timing).  Returns (tokens/s, max ms).
+    """
+    import torch
+    import torch.distributed as dist
+
+    world = dist.get_world_size() if dist.is_available() and dist.is_initialized() else 1
+    t = torch.tensor([float(ms_local)], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    ms_max = float(t.item())
+    return world * tokens_per_rank / (ms_max / 1e3), ms_max
+
+
 # ------------------------------------------------------------------ our arm
 def run_ours(args):
     import torch
@@ -318,11 +340,7 @@ def run_ours(args):
     clocks = None if args.no_clocks else sampler.stop()
     T.topk_check()
 
-    t_ms = torch.tensor([ms], device="cuda")
-    if world > 1:
-        dist.all_reduce(t_ms, op=dist.ReduceOp.MAX)
-    ms_max = float(t_ms.item())
-    value = world * w.tokens / (ms_max / 1e3)
+    value, ms_max = replica_throughput(ms, w.tokens)
 
     # end to end through the host-buffer C-ABI entry: H2D copies, call, D2H copy, every step
     e2e = None
@@ -341,10 +359,8 @@ def run_ours(args):
         for _ in range(args.e2e_steps):
             e2e_step()
         e2e_s = (time.perf_counter() - t0) / args.e2e_steps
-        te = torch.tensor([e2e_s], device="cuda")
-        if world > 1:
-            dist.all_reduce(te, op=dist.ReduceOp.MAX)
-        e2e = {"value": world * w.tokens / float(te.item()), "unit": "tokens/s", "h2d_bytes_per_step": in_bytes,
+        e2e_value, _ = replica_throughput(e2e_s * 1e3, w.tokens)
+        e2e = {"value": e2e_value, "unit": "tokens/s", "h2d_bytes_per_step": in_bytes,
                "d2h_bytes_per_step": out.numel() * out.element_size()}
 
     pk = peaks()
