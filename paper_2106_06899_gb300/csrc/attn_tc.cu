@@ -69,10 +69,10 @@ struct Layout {
   // adds up to OW/8 groups, so fewer than OW/8 + 1 does not work (0)
   static constexpr int kMinRec = TcShape<D>::OW / 8 + 1;
   static int rec_cap(int topk) {
-    const size_t heap = Sel::bytes(topk, 0);
     if (kFixed + Sel::bytes(topk, kMinRec) > kMaxSmem) return 0;
-    const size_t room = (kMaxSmem - kFixed - heap) / (BM * 44);
-    return room >= 24 ? 24 : static_cast<int>(room);
+    int gr = kMinRec;
+    while (gr < 24 && kFixed + Sel::bytes(topk, gr + 1) <= kMaxSmem) ++gr;
+    return gr;
   }
   __host__ __device__ static size_t sel_bytes(int topk, int gr) { return (Sel::bytes(topk, gr) + 15) & ~size_t(15); }
   static size_t bytes(int topk) { return kFixed + sel_bytes(topk, rec_cap(topk)); }

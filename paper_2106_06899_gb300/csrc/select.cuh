@@ -75,20 +75,23 @@ struct RowHeap {
   uint64_t root;   // heap[0] once full
   float tau;       // score of heap[0] once full, else -inf
 
-  // shared memory: heap (k + kPad) x ROWS x 8 bytes, records gr x ROWS x 36
-  // bytes, stage 8 gr x ROWS bytes (gr <= 32, so that a code fits in a byte)
+  // shared memory: heap (k + kPad) x ROWS x 8 bytes, records (gr + 1) x ROWS
+  // x 36 bytes (the last one a scratch slot), stage 8 gr x ROWS bytes (gr <=
+  // 31, so that a code fits in one byte)
   __host__ __device__ static constexpr size_t bytes(int k_, int gr_) {
-    return static_cast<size_t>(ROWS) * (static_cast<size_t>(k_ + kPad) * 8 + static_cast<size_t>(gr_) * 44);
+    return static_cast<size_t>(ROWS) *
+           (static_cast<size_t>(k_ + kPad) * 8 + static_cast<size_t>(gr_ + 1) * 36 + static_cast<size_t>(gr_) * 8);
   }
 
   __device__ __forceinline__ void init(uint8_t* smem, int row, int cap, int rec_cap) {
     base = reinterpret_cast<uint64_t*>(smem) + row;
     uint8_t* r = smem + static_cast<size_t>(cap + kPad) * ROWS * 8;
     for (int q = 0; q < kPad; ++q) base[(cap + q) * ROWS] = ~0ull;  // sentinels never leave the leaves
+    const size_t nrec = static_cast<size_t>(rec_cap) + 1;  // + scratch slot
     rlo = reinterpret_cast<float4*>(r) + row;
-    rhi = reinterpret_cast<float4*>(r + static_cast<size_t>(rec_cap) * ROWS * 16) + row;
-    rj = reinterpret_cast<uint32_t*>(r + static_cast<size_t>(rec_cap) * ROWS * 32) + row;
-    stage = r + static_cast<size_t>(rec_cap) * ROWS * 36 + row;
+    rhi = reinterpret_cast<float4*>(r + nrec * ROWS * 16) + row;
+    rj = reinterpret_cast<uint32_t*>(r + nrec * ROWS * 32) + row;
+    stage = r + nrec * ROWS * 36 + row;
     k = cap;
     gr = rec_cap;
     n = 0;
@@ -273,15 +276,17 @@ struct RowHeap {
     for (int g = 0; g < G; ++g)
       m[g] = max3f(max3f(v[8 * g], v[8 * g + 1], v[8 * g + 2]), max3f(v[8 * g + 3], v[8 * g + 4], v[8 * g + 5]),
                    fmaxf(v[8 * g + 6], v[8 * g + 7]));
+    // branch-free: a group that does not beat tau is written to the scratch
+    // slot gr (never read) and does not advance the count
     int r = rc;
 #pragma unroll
     for (int g = 0; g < G; ++g) {
-      if (m[g] > tau) {
-        rlo[r * ROWS] = make_float4(v[8 * g], v[8 * g + 1], v[8 * g + 2], v[8 * g + 3]);
-        rhi[r * ROWS] = make_float4(v[8 * g + 4], v[8 * g + 5], v[8 * g + 6], v[8 * g + 7]);
-        rj[r * ROWS] = j0 + 8 * g;
-        ++r;
-      }
+      const int pass = m[g] > tau ? 1 : 0;
+      const int slot = pass ? r : gr;
+      rlo[slot * ROWS] = make_float4(v[8 * g], v[8 * g + 1], v[8 * g + 2], v[8 * g + 3]);
+      rhi[slot * ROWS] = make_float4(v[8 * g + 4], v[8 * g + 5], v[8 * g + 6], v[8 * g + 7]);
+      rj[slot * ROWS] = j0 + 8 * g;
+      r += pass;
     }
     rc = r;
     if (__any_sync(0xffffffffu, rc > gr - G)) flush();
