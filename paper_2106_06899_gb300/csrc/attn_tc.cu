@@ -13,6 +13,15 @@
 //               key tile it sorts the k kept keys, applies the softmax over
 //               them and gathers the matching value rows (fp32 accumulate).
 //
+// Split variant (when the heaps and a record ring fit in shared memory):
+//   warps 2..5  filter: read the scores from TMEM and pass the groups of 8
+//               that beat the row's threshold into the row's record ring
+//   warps 6..9  heap: warp w serves the rows of warp w-4 (same TMEM lane
+//               quarter, same SM sub-partition); it expands the records into
+//               the heaps, publishes the rising threshold and, after the
+//               unit's last record, does the sort/softmax/gather epilogue
+//               while its filter warp already reads the next unit's scores.
+//
 // The score tile never leaves TMEM/registers: no [C x Lk] matrix is written
 // to device memory (Sec. 2.2 "Query chunking": memory O(C Lk) becomes
 // O(C k) here, in shared memory).  The scale of Eq. 1 is folded into Q by
@@ -29,31 +38,34 @@ namespace topk {
 namespace {
 
 constexpr int BM = 128;
-constexpr int kThreads = 192;
+template <bool SPLIT>
+constexpr int kThreads = SPLIT ? 320 : 192;
 
-template <int D>
+template <int D, bool SPLIT>
 struct TcShape;
-// N: keys per tile (MMA N); S: key-ring stages; OW: scores per selection call
-template <>
-struct TcShape<64> {
-  static constexpr int N = 256;
-  static constexpr int S = 2;
+// N: keys per tile (MMA N); S: key-ring stages; OW: scores per selection call.
+// The split variant takes smaller key tiles to leave room for its record ring.
+template <bool SPLIT>
+struct TcShape<64, SPLIT> {
+  static constexpr int N = SPLIT ? 128 : 256;
+  static constexpr int S = SPLIT ? 3 : 2;
   static constexpr int OW = 32;
 };
-template <>
-struct TcShape<128> {
+template <bool SPLIT>
+struct TcShape<128, SPLIT> {
   static constexpr int N = 64;
   static constexpr int S = 2;
   static constexpr int OW = 32;
 };
 
-
-
-template <int D, int FK>
+template <int D, int FK, bool SPLIT>
 struct Layout {
   using Sel = RowHeap<BM, FK>;
-  static constexpr int N = TcShape<D>::N;
-  static constexpr int S = TcShape<D>::S;
+  using Heap = HeapCore<BM, FK>;
+  using Ring = RingView<BM>;
+  static constexpr int N = TcShape<D, SPLIT>::N;
+  static constexpr int S = TcShape<D, SPLIT>::S;
+  static constexpr int OW = TcShape<D, SPLIT>::OW;
   static constexpr int R = D / 64;  // 128-byte column blocks per row
   static constexpr uint32_t Q_BYTES = BM * D * 2;
   static constexpr uint32_t KST_BYTES = N * D * 2;
@@ -65,17 +77,28 @@ struct Layout {
   static constexpr size_t kMaxSmem = 232448;
   static constexpr size_t kFixed = 1024 + OFF_SEL + CTRL_BYTES;
 
-  // pending score groups per row: as many as fit, at most 24; a selection call
-  // adds up to OW/8 groups, so fewer than OW/8 + 1 does not work (0)
-  static constexpr int kMinRec = TcShape<D>::OW / 8 + 1;
-  static int rec_cap(int topk) {
-    if (kFixed + Sel::bytes(topk, kMinRec) > kMaxSmem) return 0;
-    int gr = kMinRec;
-    while (gr < 24 && kFixed + Sel::bytes(topk, gr + 1) <= kMaxSmem) ++gr;
-    return gr;
+  // Single-warp selection: pending score groups per row, as many as fit, at
+  // most 24; a selection call adds up to OW/8 groups, so fewer than OW/8 + 1
+  // does not work (0).  Split selection: record ring slots per row, at most
+  // 24, at least two selection calls' worth.
+  static constexpr int kMinCap = SPLIT ? 2 * (OW / 8) : OW / 8 + 1;
+  __host__ __device__ static constexpr size_t heap_bytes(int topk) {
+    return (Heap::heap_bytes(topk) + 15) & ~size_t(15);
   }
-  __host__ __device__ static size_t sel_bytes(int topk, int gr) { return (Sel::bytes(topk, gr) + 15) & ~size_t(15); }
-  static size_t bytes(int topk) { return kFixed + sel_bytes(topk, rec_cap(topk)); }
+  __host__ __device__ static size_t sel_bytes(int topk, int cap) {
+    if constexpr (SPLIT)
+      return heap_bytes(topk) + ((Ring::bytes(cap) + 15) & ~size_t(15));
+    else
+      return (Sel::bytes(topk, cap) + 15) & ~size_t(15);
+  }
+  static int cap(int topk) {
+    if (kFixed + sel_bytes(topk, kMinCap) > kMaxSmem) return 0;
+    int c = kMinCap;
+    while (c < 24 && kFixed + sel_bytes(topk, c + 1) <= kMaxSmem) ++c;
+    return c;
+  }
+  static bool fits(int topk) { return cap(topk) >= kMinCap; }
+  static size_t bytes(int topk) { return kFixed + sel_bytes(topk, cap(topk)); }
 };
 
 // Waits on an mbarrier phase with lane 0 of the warp and broadcasts the
@@ -100,13 +123,13 @@ __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, const
   }
 }
 
-template <int D, int FK>
-__global__ void __launch_bounds__(kThreads, 1)
+template <int D, int FK, bool SPLIT>
+__global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmk,
                    const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ out, int BH, int Lq, int Lk,
-                   int topk, int rec_cap, int causal, int n_units, int32_t* __restrict__ idx,
-                   float* __restrict__ score, DevCtl ctl) {
-  using L = Layout<D, FK>;
+                   int topk, int rec_cap, int causal, int n_units, int pre_keys, int pre_group,
+                   int32_t* __restrict__ idx, float* __restrict__ score, DevCtl ctl) {
+  using L = Layout<D, FK, SPLIT>;
   using Sel = typename L::Sel;
   constexpr int N = L::N, S = L::S, R = L::R;
   constexpr uint32_t IDESC = idesc_bf16_f32(BM, N);
@@ -117,6 +140,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* q_s = smem + L::OFF_Q;
   uint8_t* k_s = smem + L::OFF_K;
   uint8_t* sel_mem = smem + L::OFF_SEL;
+  uint8_t* ring_mem = sel_mem + L::heap_bytes(topk);  // split variant only
   uint64_t* bars = reinterpret_cast<uint64_t*>(sel_mem + L::sel_bytes(topk, rec_cap));
   uint64_t* full_k = bars;
   uint64_t* empty_k = bars + S;
@@ -146,6 +170,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
+  if constexpr (SPLIT) {  // ring counters, end marks and thresholds start at 0
+    uint32_t* z = reinterpret_cast<uint32_t*>(ring_mem);
+    for (int i = threadIdx.x; i < static_cast<int>(L::Ring::ctl_bytes() / 4); i += blockDim.x) z[i] = 0;
+  }
   if (warp == 1) tmem_alloc(tmem_slot, TMEM_COLS);
   tc_fence_before();
   __syncthreads();
@@ -165,6 +193,15 @@ __global__ void __launch_bounds__(kThreads, 1)
   auto key_tiles = [&](int qt) {
     const int kend = causal ? min(Lk, (qt + 1) * BM) : Lk;
     return (kend + N - 1) / N;
+  };
+  // Floor pre-pass (split variant): the first pre_keys keys are scored once
+  // more ahead of the unit, in topk groups of pre_group keys; the smallest
+  // group maximum is a floor of the row's k-th largest score.  Only where it
+  // costs at most an eighth of the unit's keys.
+  auto pre_tiles = [&](int qt) {
+    if (pre_group == 0) return 0;
+    const int kend = causal ? min(Lk, (qt + 1) * BM) : Lk;
+    return kend / 8 >= pre_keys ? (pre_keys + N - 1) / N : 0;
   };
 
   if (warp == 0) {
@@ -187,8 +224,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int r = 0; r < R; ++r) tma_load_3d(q_s + r * BM * 128, &tmq, q_full, r * 64, qt * BM, bh);
       }
       ++q_issued;
-      const int nk = key_tiles(qt);
-      for (int kt = 0; kt < nk; ++kt) {
+      const int npre = pre_tiles(qt);
+      const int nk = npre + key_tiles(qt);
+      for (int t = 0; t < nk; ++t) {
+        const int kt = t < npre ? t : t - npre;
         const int s = it % S;
         const uint32_t ph = (it / S) & 1u;
         if (!warp_wait(&empty_k[s], ph ^ 1u, ctl, abort_flag)) {
@@ -230,7 +269,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       tc_fence_after();
-      const int nk = key_tiles(qt);
+      const int nk = pre_tiles(qt) + key_tiles(qt);
       for (int kt = 0; kt < nk; ++kt, ++it, ++acc_it) {
         const int s = it % S;
         if (!warp_wait(&full_k[s], (it / S) & 1u, ctl, abort_flag)) {
@@ -268,6 +307,131 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_drain(drain, 0, ctl);
     }
     __syncwarp();
+  } else if (SPLIT && warp < 6) {
+    // ------------------------------------------------------------ filter (split)
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
+    constexpr int OW = L::OW;
+    uint32_t acc_it = 0;
+    RowFilter<BM> f;
+    f.init(ring_mem, row, rec_cap);
+    bool ok = true;
+    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
+      int bh, qt;
+      decode(u, bh, qt);
+      f.begin_unit();
+      const int i_row = qt * BM + row;
+      const int nk = key_tiles(qt);
+      const int npre = pre_tiles(qt);
+      const uint32_t lim = static_cast<uint32_t>(causal ? min(i_row + 1, Lk) : Lk);
+      const int lim_min = causal ? min(qt * BM + 1, Lk) : Lk;
+      if (npre > 0) {
+        // pre-pass: F = min over the topk groups of their maxima (masked
+        // keys are -inf, so a row with a short key range gets no floor)
+        float F = INFINITY, gm = -INFINITY;
+        for (int kt = 0; ok && kt < npre; ++kt, ++acc_it) {
+          const int b = acc_it & 1;
+          if (!warp_wait(&acc_full[b], (acc_it >> 1) & 1u, ctl, abort_flag)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(b * N);
+#pragma unroll 1
+          for (int c = 0; c < N / 64; ++c) {
+            float vals[64];
+            __syncwarp();
+            tmem_ld64(taddr + c * 64, vals);
+            tmem_wait_ld();
+            if (c == N / 64 - 1) {
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(&acc_empty[b]);
+            }
+            const uint32_t j0 = static_cast<uint32_t>(kt * N + c * 64);
+            if (static_cast<int>(j0) + 64 > lim_min) mask_scores(vals, j0, lim);
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+              const uint32_t jh = j0 + 32u * h;
+              if (jh < static_cast<uint32_t>(pre_keys)) {
+                float hm = vals[32 * h];
+#pragma unroll
+                for (int e = 1; e < 31; e += 2) hm = max3f(hm, vals[32 * h + e], vals[32 * h + e + 1]);
+                hm = fmaxf(hm, vals[32 * h + 31]);
+                gm = fmaxf(gm, hm);
+                if (((jh + 32u) & static_cast<uint32_t>(pre_group - 1)) == 0u) {
+                  F = fminf(F, gm);
+                  gm = -INFINITY;
+                }
+              }
+            }
+          }
+        }
+        if (!ok) break;
+        f.set_floor(F);
+      }
+      for (int kt = 0; ok && kt < nk; ++kt, ++acc_it) {
+        const int b = acc_it & 1;
+        if (!warp_wait(&acc_full[b], (acc_it >> 1) & 1u, ctl, abort_flag)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(b * N);
+        const uint32_t jt = static_cast<uint32_t>(kt * N);
+#pragma unroll 1
+        for (int c = 0; c < N / 64; ++c) {
+          float vals[64];
+          f.refresh_tau();
+          __syncwarp();
+          tmem_ld64(taddr + c * 64, vals);
+          tmem_wait_ld();
+          if (c == N / 64 - 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&acc_empty[b]);
+          }
+          const uint32_t j0 = jt + static_cast<uint32_t>(c * 64);
+          if (static_cast<int>(j0) + 64 > lim_min) mask_scores(vals, j0, lim);
+#pragma unroll
+          for (int h = 0; h < 64 / OW; ++h) {
+            if (!f.reserve(OW / 8, ctl, abort_flag)) {
+              ok = false;
+              break;
+            }
+            f.offer(reinterpret_cast<const float(&)[OW]>(vals[h * OW]), j0 + static_cast<uint32_t>(h * OW));
+          }
+          if (!ok) break;
+          f.publish();
+        }
+      }
+      if (ok && !f.end_unit(ctl, abort_flag)) ok = false;
+    }
+  } else if (SPLIT) {
+    // ------------------------------------------------------------ heap (split)
+    const int quad = warp & 3;
+    const int row = quad * 32 + lane;
+    RowSink<BM, FK> heap;
+    heap.init(ring_mem, row, rec_cap);
+    for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
+      int bh, qt;
+      decode(u, bh, qt);
+      const int i_row = qt * BM + row;
+      heap.begin_unit(sel_mem, row, topk);
+      // batch threshold: half the ring, below the filter's margin of OW/8
+      // free slots, so that the filter never waits on a heap warp that waits
+      if (!heap.drain_unit(rec_cap / 2, ctl, abort_flag)) break;
+      if (i_row < Lq) {
+        const size_t orow = static_cast<size_t>(bh) * Lq + i_row;
+        // the softmax needs no order; only the index/score outputs are sorted
+        if (idx || score) heap.sort();
+        softmax_gather_store<__nv_bfloat16, D>(heap, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
+        if (idx || score)
+          write_selection(heap, idx ? idx + orow * topk : nullptr, score ? score + orow * topk : nullptr);
+      }
+      __syncwarp();
+    }
   } else {
     // ------------------------------------------------------------ selection
     const int quad = warp & 3;
@@ -306,7 +470,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           const uint32_t j0 = jt + static_cast<uint32_t>(c * 64);
           if (static_cast<int>(j0) + 64 > lim_min) mask_scores(vals, j0, lim);
-          constexpr int OW = TcShape<D>::OW;
+          constexpr int OW = L::OW;
 #pragma unroll
           for (int h = 0; h < 64 / OW; ++h)
             heap.offer(reinterpret_cast<const float(&)[OW]>(vals[h * OW]), j0 + static_cast<uint32_t>(h * OW));
@@ -332,9 +496,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-template <int D, int FK>
+template <int D, int FK, bool SPLIT>
 int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
-  using L = Layout<D, FK>;
+  using L = Layout<D, FK, SPLIT>;
   const int BH = a.B * a.H;
   CUtensorMap tmq, tmk;
   if (!make_tmap_bf16_3d(&tmq, a.q, D, a.Lq, BH, BM)) return -1;
@@ -344,30 +508,41 @@ int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t 
   // all TMEM columns it needs for its whole (persistent) lifetime.
   const size_t need = L::bytes(a.topk);
   const size_t smem = need > 120 * 1024 ? need : 120 * 1024;
-  auto kern = attn_tc_kernel<D, FK>;
+  auto kern = attn_tc_kernel<D, FK, SPLIT>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
       cudaSuccess)
     return -1;
   const int grid = n_units < num_sms ? n_units : num_sms;
-  kern<<<grid, kThreads, smem, st>>>(tmq, tmk, static_cast<const __nv_bfloat16*>(a.v),
-                                     static_cast<__nv_bfloat16*>(a.out), BH, a.Lq, a.Lk, a.topk,
-                                     L::rec_cap(a.topk), a.causal, n_units, a.idx, a.score, ctl);
+  // floor pre-pass (split only): topk groups of the largest power of two
+  // >= 64 keys such that the pre-pass reads at most Lk / 8 keys
+  int pre_keys = 0, pre_group = 0;
+  if (SPLIT)
+    for (long long gs = 64; static_cast<long long>(a.topk) * gs * 8 <= a.Lk; gs *= 2) {
+      pre_group = static_cast<int>(gs);
+      pre_keys = static_cast<int>(a.topk * gs);
+    }
+  kern<<<grid, kThreads<SPLIT>, smem, st>>>(tmq, tmk, static_cast<const __nv_bfloat16*>(a.v),
+                                            static_cast<__nv_bfloat16*>(a.out), BH, a.Lq, a.Lk, a.topk,
+                                            L::cap(a.topk), a.causal, n_units, pre_keys, pre_group, a.idx,
+                                            a.score, ctl);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
+// Split selection where its heaps and rings fit; the 8-ary heap for k = 64.
 template <int D>
 int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
-  if (a.topk == 64 && Layout<D, 64>::rec_cap(64) >= Layout<D, 64>::kMinRec)
-    return launch_tc_k<D, 64>(a, ctl, num_sms, st);
-  return launch_tc_k<D, 0>(a, ctl, num_sms, st);
+  if (a.topk == 64 && Layout<D, 64, true>::fits(64)) return launch_tc_k<D, 64, true>(a, ctl, num_sms, st);
+  if (Layout<D, 0, true>::fits(a.topk)) return launch_tc_k<D, 0, true>(a, ctl, num_sms, st);
+  if (a.topk == 64 && Layout<D, 64, false>::fits(64)) return launch_tc_k<D, 64, false>(a, ctl, num_sms, st);
+  return launch_tc_k<D, 0, false>(a, ctl, num_sms, st);
 }
 
 }  // namespace
 
 bool attn_tc_supports(const AttnArgs& a) {
   if (a.dtype != 1 || a.topk > kTcMaxK) return false;
-  if (a.d == 64) return Layout<64, 0>::rec_cap(a.topk) >= Layout<64, 0>::kMinRec;
-  if (a.d == 128) return Layout<128, 0>::rec_cap(a.topk) >= Layout<128, 0>::kMinRec;
+  if (a.d == 64) return Layout<64, 0, false>::fits(a.topk);
+  if (a.d == 128) return Layout<128, 0, false>::fits(a.topk);
   return false;
 }
 

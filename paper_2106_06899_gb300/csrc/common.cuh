@@ -88,6 +88,75 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const 
   }
 }
 
+// ---------------------------------------------------------------- CTA-scope
+// release/acquire on shared memory: a producer writes its data, then
+// publishes a counter with a release store; a consumer reads the counter
+// with an acquire load and then sees the data.
+__device__ __forceinline__ void st_release_u32(uint32_t* p, uint32_t v) {
+  asm volatile("st.release.cta.shared::cta.u32 [%0], %1;" ::"r"(smem_u32(p)), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ void st_release_u64(uint64_t* p, uint64_t v) {
+  asm volatile("st.release.cta.shared::cta.u64 [%0], %1;" ::"r"(smem_u32(p)), "l"(v) : "memory");
+}
+
+__device__ __forceinline__ uint32_t ld_acquire_u32(const uint32_t* p) {
+  uint32_t v;
+  asm volatile("ld.acquire.cta.shared::cta.u32 %0, [%1];" : "=r"(v) : "r"(smem_u32(p)) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ uint64_t ld_acquire_u64(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.acquire.cta.shared::cta.u64 %0, [%1];" : "=l"(v) : "r"(smem_u32(p)) : "memory");
+  return v;
+}
+
+// Predicated shared-memory stores (no branch, no write when p is false).
+__device__ __forceinline__ void st_shared_f4_if(bool p, float4* dst, float a, float b, float c, float d) {
+  asm volatile(
+      "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t"
+      "@q st.shared.v4.f32 [%1], {%2, %3, %4, %5};\n\t}" ::"r"(static_cast<int>(p)),
+      "r"(smem_u32(dst)), "f"(a), "f"(b), "f"(c), "f"(d));
+}
+
+__device__ __forceinline__ void st_shared_u32_if(bool p, uint32_t* dst, uint32_t v) {
+  asm volatile(
+      "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t"
+      "@q st.shared.u32 [%1], %2;\n\t}" ::"r"(static_cast<int>(p)),
+      "r"(smem_u32(dst)), "r"(v));
+}
+
+__device__ __forceinline__ void st_shared_u2_if(bool p, uint2* dst, uint32_t a, uint32_t b) {
+  asm volatile(
+      "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t"
+      "@q st.shared.v2.u32 [%1], {%2, %3};\n\t}" ::"r"(static_cast<int>(p)),
+      "r"(smem_u32(dst)), "r"(a), "r"(b)
+      : "memory");
+}
+
+// Predicated 64-bit store that also orders the compiler's memory accesses
+// around it (the same thread reads the slot back later).
+__device__ __forceinline__ void st_shared_u64_if(bool p, uint64_t* dst, uint64_t v) {
+  asm volatile(
+      "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t"
+      "@q st.shared.u64 [%1], %2;\n\t}" ::"r"(static_cast<int>(p)),
+      "r"(smem_u32(dst)), "l"(v)
+      : "memory");
+}
+
+// Relaxed load: a value that only ever grows (a threshold), read without
+// ordering the surrounding accesses.
+__device__ __forceinline__ uint64_t ld_relaxed_u64(const uint64_t* p) {
+  uint64_t v;
+  asm volatile("ld.relaxed.cta.shared::cta.u64 %0, [%1];" : "=l"(v) : "r"(smem_u32(p)));
+  return v;
+}
+
+__device__ __forceinline__ void st_relaxed_u64(uint64_t* p, uint64_t v) {
+  asm volatile("st.relaxed.cta.shared::cta.u64 [%0], %1;" ::"r"(smem_u32(p)), "l"(v));
+}
+
 // ---------------------------------------------------------------- TMA
 __device__ __forceinline__ void tma_prefetch_desc(const void* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");

@@ -41,61 +41,43 @@ __device__ __forceinline__ float key_score(uint64_t key) { return unord_f32(stat
 
 __device__ __forceinline__ uint32_t key_index(uint64_t key) { return ~static_cast<uint32_t>(key); }
 
-// Exact per-row top-k: a 4-ary min-heap of packed keys in shared memory,
-// fed through a per-row buffer of pending score groups.
-//
-// The filter compares the maximum of each group of 8 scores with tau (the
-// heap root's score, -inf until the heap is full) and, if it wins, copies
-// the whole group (8 scores and its first key index) into the row's record
-// buffer with two vector stores: no per-element work and no loop on the
-// divergent path.  When any lane of the warp has filled its record buffer,
-// the whole warp expands its records into the heaps in lockstep (flush):
-// elements are offered in ascending key index, each one that beats the
-// current root replaces it.  tau only rises, so records taken against a
-// stale tau can hold a few elements that no longer qualify; they are
-// re-checked at expansion.  The 4-ary heap halves the dependent shared
-// memory round trips of a replace (log4 k levels of four independent loads).
-// ROWS = number of rows sharing the [slot][row] arrays (the row stride);
-// every call of offer*/flush/finish must be made by all 32 lanes of a warp.
+// The largest float below s (s itself if it is -inf): x > below_f32(s)
+// exactly when x >= s, for any float x that is not NaN.  -0 is skipped: it
+// compares equal to +0, so the float below +0 is the negative denormal of
+// least magnitude.
+__device__ __forceinline__ float below_f32(float s) {
+  if (s == -INFINITY) return s;
+  uint32_t o = ord_f32(s) - 1u;
+  if (o == 0x7FFFFFFFu) o -= 1u;
+  return unord_f32(o);
+}
+
+// The heap of one row: a min-heap of its k best packed keys in shared memory
+// ([slot][row] layout, ROWS rows per slot).  push() offers one key; sort()
+// turns the heap into the kept keys in selection order.  The 4-ary layout
+// halves the dependent shared-memory round trips of a replace (log4 k levels
+// of four independent loads).
 template <int ROWS, int FIXED_K = 0>
-struct RowHeap {
+struct HeapCore {
   // FIXED_K == 64: an 8-ary heap of exactly 64 keys, padded with 9 sentinel
   // slots (largest key) so that every interior node has 8 children: a root
   // replacement is two fully unrolled levels of 8 independent loads.
   static constexpr int kPad = FIXED_K == 64 ? 9 : 0;
   uint64_t* base;  // &heap[slot 0][this row]
-  float4* rlo;     // &records_lo[0][this row]: scores 0..3
-  float4* rhi;     // &records_hi[0][this row]: scores 4..7
-  uint32_t* rj;    // &records_j0[0][this row]
-  uint8_t* stage;  // &stage[0][this row]: codes (record slot * 8 + element) of elements to offer
   int k;           // capacity
   int n;           // entries filled
-  int rc;          // records pending
-  int gr;          // record capacity
   uint64_t root;   // heap[0] once full
   float tau;       // score of heap[0] once full, else -inf
 
-  // shared memory: heap (k + kPad) x ROWS x 8 bytes, records (gr + 1) x ROWS
-  // x 36 bytes (the last one a scratch slot), stage 8 gr x ROWS bytes (gr <=
-  // 31, so that a code fits in one byte)
-  __host__ __device__ static constexpr size_t bytes(int k_, int gr_) {
-    return static_cast<size_t>(ROWS) *
-           (static_cast<size_t>(k_ + kPad) * 8 + static_cast<size_t>(gr_ + 1) * 36 + static_cast<size_t>(gr_) * 8);
+  __host__ __device__ static constexpr size_t heap_bytes(int k_) {
+    return static_cast<size_t>(ROWS) * static_cast<size_t>(k_ + kPad) * 8;
   }
 
-  __device__ __forceinline__ void init(uint8_t* smem, int row, int cap, int rec_cap) {
+  __device__ __forceinline__ void init_heap(uint8_t* smem, int row, int cap) {
     base = reinterpret_cast<uint64_t*>(smem) + row;
-    uint8_t* r = smem + static_cast<size_t>(cap + kPad) * ROWS * 8;
     for (int q = 0; q < kPad; ++q) base[(cap + q) * ROWS] = ~0ull;  // sentinels never leave the leaves
-    const size_t nrec = static_cast<size_t>(rec_cap) + 1;  // + scratch slot
-    rlo = reinterpret_cast<float4*>(r) + row;
-    rhi = reinterpret_cast<float4*>(r + nrec * ROWS * 16) + row;
-    rj = reinterpret_cast<uint32_t*>(r + nrec * ROWS * 32) + row;
-    stage = r + nrec * ROWS * 36 + row;
     k = cap;
-    gr = rec_cap;
     n = 0;
-    rc = 0;
     root = 0;
     tau = -INFINITY;
   }
@@ -135,10 +117,13 @@ struct RowHeap {
   }
 
   // 8-ary heap of 64 keys: children of node p are 8p+1 .. 8p+8; slots 64..72
-  // hold sentinels.  Replace the root by x and restore the heap order.
-  __device__ __forceinline__ void replace_root64(uint64_t x) {
+  // hold sentinels.  Replace the root by x and restore the heap order;
+  // returns the new root (the smaller of x and the root's smallest child),
+  // so that the caller need not read it back.
+  __device__ __forceinline__ uint64_t replace_root64(uint64_t x) {
     int p = 0;
     bool done = false;
+    uint64_t new_root = x;
 #pragma unroll
     for (int level = 0; level < 2; ++level) {
       const int c = 8 * p + 1;
@@ -160,6 +145,7 @@ struct RowHeap {
       const bool lf = m01 <= m23;
       const uint64_t a = lf ? m01 : m23;
       const int ca = c + (lf ? i01 : i23);
+      if (level == 0 && a < x) new_root = a;
       if (!done && a < x) {
         put(p, a);
         p = ca;
@@ -168,6 +154,53 @@ struct RowHeap {
       }
     }
     put(p, x);
+    return new_root;
+  }
+
+  // Branch-free form of replace_root64 for a full 8-ary heap of 64: if act,
+  // x (which must rank above the root) replaces the root; both levels are
+  // always read and the stores are predicated, so that a warp whose lanes
+  // disagree on act runs one straight-line body.  Returns the root after
+  // the call (`cur`, the current root, when act is false).
+  __device__ __forceinline__ uint64_t replace_root64_pred(uint64_t x, bool act, uint64_t cur) {
+    uint64_t ch[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) ch[q] = get(1 + q);
+    uint64_t a0;
+    int i0;
+    argmin8(ch, a0, i0);
+    const int c0 = 1 + i0;
+    const bool go0 = act && a0 < x;
+    const int c1b = 8 * c0 + 1;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) ch[q] = get(c1b + q);
+    uint64_t a1;
+    int i1;
+    argmin8(ch, a1, i1);
+    const bool go1 = go0 && a1 < x;
+    const uint64_t top = go0 ? a0 : x;
+    st_shared_u64_if(act, base, top);
+    st_shared_u64_if(go0, base + c0 * ROWS, go1 ? a1 : x);
+    st_shared_u64_if(go1, base + (c1b + i1) * ROWS, x);
+    return act ? top : cur;
+  }
+
+  // Smallest of 8 keys and its position (tree of depth 3).
+  __device__ __forceinline__ static void argmin8(const uint64_t (&ch)[8], uint64_t& m, int& i) {
+    uint64_t m2[4];
+    int i2[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const bool lo = ch[2 * q] <= ch[2 * q + 1];
+      m2[q] = lo ? ch[2 * q] : ch[2 * q + 1];
+      i2[q] = lo ? 2 * q : 2 * q + 1;
+    }
+    const bool l01 = m2[0] <= m2[1], l23 = m2[2] <= m2[3];
+    const uint64_t m01 = l01 ? m2[0] : m2[1], m23 = l23 ? m2[2] : m2[3];
+    const int i01 = l01 ? i2[0] : i2[1], i23 = l23 ? i2[2] : i2[3];
+    const bool lf = m01 <= m23;
+    m = lf ? m01 : m23;
+    i = lf ? i01 : i23;
   }
 
   // Add x: while the heap is not full it is appended (the heap is built
@@ -189,11 +222,11 @@ struct RowHeap {
       }
     } else if (x > root) {
       if constexpr (FIXED_K == 64) {
-        replace_root64(x);
+        root = replace_root64(x);
       } else {
         sift_down(x, 0, k);
+        root = get(0);
       }
-      root = get(0);
       tau = key_score(root);
     }
   }
@@ -218,6 +251,79 @@ struct RowHeap {
       p = ca;
     }
     put(p, x);
+  }
+
+  // Heap-sort in place so that slots 0 .. n-1 hold the kept keys in
+  // selection order (best first).  A row that never filled its heap (fewer
+  // than k valid keys) is heapified first: its entries were appended
+  // unordered.
+  __device__ __forceinline__ void sort() {
+    if constexpr (FIXED_K == 64) {
+      if (n < k && n > 1)
+        for (int p = (n - 2) / 8; p >= 0; --p) sift_down8(get(p), p, n);
+      for (int m = n - 1; m > 0; --m) {
+        const uint64_t x = get(m);
+        put(m, get(0));
+        sift_down8(x, 0, m);
+      }
+    } else {
+      if (n < k && n > 1)
+        for (int p = (n - 2) / 4; p >= 0; --p) sift_down(get(p), p, n);
+      for (int m = n - 1; m > 0; --m) {
+        const uint64_t x = get(m);
+        put(m, get(0));
+        sift_down(x, 0, m);
+      }
+    }
+  }
+};
+
+// Exact per-row top-k for one warp that both filters and keeps the heap:
+// HeapCore fed through a per-row buffer of pending score groups.
+//
+// The filter compares the maximum of each group of 8 scores with tau (the
+// heap root's score, -inf until the heap is full) and, if it wins, copies
+// the whole group (8 scores and its first key index) into the row's record
+// buffer with two vector stores: no per-element work and no loop on the
+// divergent path.  When any lane of the warp has filled its record buffer,
+// the whole warp expands its records into the heaps in lockstep (flush):
+// elements are offered in ascending key index, each one that beats the
+// current root replaces it.  tau only rises, so records taken against a
+// stale tau can hold a few elements that no longer qualify; they are
+// re-checked at expansion.
+// ROWS = number of rows sharing the [slot][row] arrays (the row stride);
+// every call of offer*/flush/finish must be made by all 32 lanes of a warp.
+template <int ROWS, int FIXED_K = 0>
+struct RowHeap : HeapCore<ROWS, FIXED_K> {
+  using Core = HeapCore<ROWS, FIXED_K>;
+  using Core::kPad;
+  using Core::push;
+  using Core::tau;
+  float4* rlo;     // &records_lo[0][this row]: scores 0..3
+  float4* rhi;     // &records_hi[0][this row]: scores 4..7
+  uint32_t* rj;    // &records_j0[0][this row]
+  uint8_t* stage;  // &stage[0][this row]: codes (record slot * 8 + element) of elements to offer
+  int rc;          // records pending
+  int gr;          // record capacity
+
+  // shared memory: heap (k + kPad) x ROWS x 8 bytes, records (gr + 1) x ROWS
+  // x 36 bytes (the last one a scratch slot), stage 8 gr x ROWS bytes (gr <=
+  // 31, so that a code fits in one byte)
+  __host__ __device__ static constexpr size_t bytes(int k_, int gr_) {
+    return Core::heap_bytes(k_) +
+           static_cast<size_t>(ROWS) * (static_cast<size_t>(gr_ + 1) * 36 + static_cast<size_t>(gr_) * 8);
+  }
+
+  __device__ __forceinline__ void init(uint8_t* smem, int row, int cap, int rec_cap) {
+    Core::init_heap(smem, row, cap);
+    uint8_t* r = smem + Core::heap_bytes(cap);
+    const size_t nrec = static_cast<size_t>(rec_cap) + 1;  // + scratch slot
+    rlo = reinterpret_cast<float4*>(r) + row;
+    rhi = reinterpret_cast<float4*>(r + nrec * ROWS * 16) + row;
+    rj = reinterpret_cast<uint32_t*>(r + nrec * ROWS * 32) + row;
+    stage = r + nrec * ROWS * 36 + row;
+    gr = rec_cap;
+    rc = 0;
   }
 
   // Expand every lane's pending records into its heap, in two phases.
@@ -292,28 +398,328 @@ struct RowHeap {
     if (__any_sync(0xffffffffu, rc > gr - G)) flush();
   }
 
-  // After the last key: merge what is pending, then heap-sort in place so
-  // that slots 0 .. n-1 hold the kept keys in selection order (best first).
-  // A row that never filled its heap (fewer than k valid keys) is heapified
-  // first: its entries were appended unordered.
+  // After the last key: merge what is pending, then sort.
   __device__ __forceinline__ void finish() {
     flush();
-    if constexpr (FIXED_K == 64) {
-      if (n < k && n > 1)
-        for (int p = (n - 2) / 8; p >= 0; --p) sift_down8(get(p), p, n);
-      for (int m = n - 1; m > 0; --m) {
-        const uint64_t x = get(m);
-        put(m, get(0));
-        sift_down8(x, 0, m);
+    Core::sort();
+  }
+};
+
+// ---------------------------------------------------------------------------
+// Split selection: a filter warp and a heap warp share the same 32 rows.
+//
+// The filter warp reads the scores and keeps no heap: each group of 8 whose
+// maximum beats its copy of the row's threshold goes, as one record (8 scores
+// and the first key index), into the row's ring of R records.  The heap warp
+// expands the records into the row's heap exactly as RowHeap::flush does and
+// publishes the heap root's score as the new threshold.  Both warps run on
+// the same SM sub-partition, so the heap work of one batch overlaps the
+// filtering of the next instead of following it.
+//
+// Per row, in shared memory ([slot][row] like the heap):
+//   end   u64  (unit sequence number << 32) | head at the unit's last record
+//   tauw  u64  (unit sequence number << 32) | bits of the heap root's score
+//   head  u32  records written (filter, release store)
+//   tail  u32  records consumed (heap warp, release store)
+//   flw   u64  (unit sequence number << 32) | bits of a score floor that the
+//              filter found before its first record (a pre-pass), or 0
+//   R record slots, then kStage (score, index) pairs: the heap warp's own
+//   list of the elements it is about to offer to the heap.  The heap warp
+//   copies the qualifying elements out of the records first and frees the
+//   slots at once, so that the filter refills the ring while the heap works.
+// Counters are absolute and wrap modulo 2^32; the slot of record number c is
+// c mod R (tracked incrementally).  Each unit (query tile) has a sequence
+// number 1, 2, ... per CTA; a threshold or end mark of another unit is
+// ignored.
+template <int ROWS>
+struct RingView {
+  static constexpr int kStage = 24;
+  uint64_t* end;
+  uint64_t* tauw;
+  uint32_t* head;
+  uint32_t* tail;
+  uint64_t* flw;
+  float4* lo;
+  float4* hi;
+  uint32_t* rj;
+  uint2* stage;
+
+  __host__ __device__ static constexpr size_t ctl_bytes() { return static_cast<size_t>(ROWS) * 32; }
+  __host__ __device__ static constexpr size_t bytes(int R) {
+    return ctl_bytes() + static_cast<size_t>(ROWS) * (static_cast<size_t>(R) * 36 + kStage * 8);
+  }
+
+  // mem must be 16-byte aligned; its first ctl_bytes() must be zero before use
+  __device__ __forceinline__ void bind(uint8_t* mem, int row, int R) {
+    end = reinterpret_cast<uint64_t*>(mem) + row;
+    tauw = reinterpret_cast<uint64_t*>(mem + ROWS * 8) + row;
+    head = reinterpret_cast<uint32_t*>(mem + ROWS * 16) + row;
+    tail = reinterpret_cast<uint32_t*>(mem + ROWS * 20) + row;
+    flw = reinterpret_cast<uint64_t*>(mem + ROWS * 24) + row;
+    uint8_t* r = mem + ctl_bytes();
+    const size_t nrec = static_cast<size_t>(R);
+    lo = reinterpret_cast<float4*>(r) + row;
+    hi = reinterpret_cast<float4*>(r + nrec * ROWS * 16) + row;
+    stage = reinterpret_cast<uint2*>(r + nrec * ROWS * 32) + row;
+    rj = reinterpret_cast<uint32_t*>(r + nrec * ROWS * 32 + kStage * ROWS * 8) + row;
+  }
+};
+
+// Sleep between polls of a shared-memory counter: doubles from 32 ns to 512
+// ns, so that a waiting warp leaves the issue slots of its SM sub-partition
+// to the warp it waits for.
+__device__ __forceinline__ unsigned backoff_ns(uint32_t polls) { return 32u << (polls < 4u ? polls : 4u); }
+
+// Filter side.  Every call is made by all 32 lanes of the warp.
+template <int ROWS>
+struct RowFilter {
+  RingView<ROWS> v;
+  int R;
+  uint32_t h;    // records written
+  int hm;        // h mod R
+  uint32_t tc;   // last tail seen
+  uint32_t seq;  // current unit
+  float tau;     // threshold: a lower bound of the row's final k-th score
+
+  __device__ __forceinline__ void init(uint8_t* mem, int row, int R_) {
+    v.bind(mem, row, R_);
+    R = R_;
+    h = 0;
+    hm = 0;
+    tc = 0;
+    seq = 0;
+  }
+
+  __device__ __forceinline__ void begin_unit() {
+    ++seq;
+    tau = -INFINITY;
+  }
+
+  // Adopt the heap warp's threshold if it belongs to this unit.
+  __device__ __forceinline__ void refresh_tau() {
+    const uint64_t w = ld_relaxed_u64(v.tauw);
+    if (static_cast<uint32_t>(w >> 32) == seq) tau = fmaxf(tau, __uint_as_float(static_cast<uint32_t>(w)));
+  }
+
+  // Waits (bounded) until every lane has room for `need` more records.
+  // Everything written so far is published first: the heap warp may be
+  // waiting for a fuller batch than it can see.
+  __device__ __forceinline__ bool reserve(int need, const DevCtl& ctl, volatile int* abort_flag) {
+    if (__all_sync(0xffffffffu, static_cast<int>(h - tc) + need <= R)) return true;
+    publish();
+    unsigned long long t0 = 0;
+    for (uint32_t spin = 0;; ++spin) {
+      tc = ld_acquire_u32(v.tail);
+      if (__all_sync(0xffffffffu, static_cast<int>(h - tc) + need <= R)) return true;
+      int stop = 0;
+      if ((threadIdx.x & 31) == 0 && (spin & 15u) == 0) {
+        if (spin == 0) {
+          t0 = global_ns();
+        } else if (*abort_flag) {
+          stop = 1;
+        } else if (global_ns() - t0 > ctl.wait_limit_ns) {
+          atomicOr(ctl.error, kDevErrTimeout);
+          *abort_flag = 1;
+          stop = 1;
+        }
       }
+      if (__shfl_sync(0xffffffffu, stop, 0)) return false;
+      __nanosleep(backoff_ns(spin));
+    }
+  }
+
+  // Offer W scores with key indices j0 .. j0+W-1; needs W/8 free slots.
+  // A group that does not pass costs no shared-memory store (predicated).
+  template <int W>
+  __device__ __forceinline__ void offer(const float (&x)[W], uint32_t j0) {
+    constexpr int G = W / 8;
+    float m[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g)
+      m[g] = max3f(max3f(x[8 * g], x[8 * g + 1], x[8 * g + 2]), max3f(x[8 * g + 3], x[8 * g + 4], x[8 * g + 5]),
+                   fmaxf(x[8 * g + 6], x[8 * g + 7]));
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+      const bool pass = m[g] > tau;
+      st_shared_f4_if(pass, v.lo + hm * ROWS, x[8 * g], x[8 * g + 1], x[8 * g + 2], x[8 * g + 3]);
+      st_shared_f4_if(pass, v.hi + hm * ROWS, x[8 * g + 4], x[8 * g + 5], x[8 * g + 6], x[8 * g + 7]);
+      st_shared_u32_if(pass, v.rj + hm * ROWS, j0 + 8 * g);
+      const int nx = hm + (pass ? 1 : 0);
+      hm = nx == R ? 0 : nx;
+      h += pass ? 1u : 0u;
+    }
+  }
+
+  // Adopt a floor F of the row's k-th largest score (at least k scores of
+  // the row are >= F): from now on only scores >= F pass, and the heap warp
+  // applies the same floor while its heap is filling.  Called before the
+  // unit's first record.
+  __device__ __forceinline__ void set_floor(float F) {
+    const float below = below_f32(F);  // x > below  <=>  x >= F
+    tau = fmaxf(tau, below);
+    st_release_u64(v.flw, (static_cast<uint64_t>(seq) << 32) | __float_as_uint(below));
+  }
+
+  // Make the records written so far visible to the heap warp.
+  __device__ __forceinline__ void publish() { st_release_u32(v.head, h); }
+
+  // Mark the end of this unit's records.  The heap warp must have taken the
+  // previous unit's end mark first (it says so by publishing a threshold word
+  // of this unit when it starts it): the end word has one slot.
+  __device__ __forceinline__ bool end_unit(const DevCtl& ctl, volatile int* abort_flag) {
+    unsigned long long t0 = 0;
+    for (uint32_t spin = 0;; ++spin) {
+      const uint32_t s = static_cast<uint32_t>(ld_acquire_u64(v.tauw) >> 32);
+      if (__all_sync(0xffffffffu, s == seq)) break;
+      int stop = 0;
+      if ((threadIdx.x & 31) == 0 && (spin & 15u) == 0) {
+        if (spin == 0) {
+          t0 = global_ns();
+        } else if (*abort_flag) {
+          stop = 1;
+        } else if (global_ns() - t0 > ctl.wait_limit_ns) {
+          atomicOr(ctl.error, kDevErrTimeout);
+          *abort_flag = 1;
+          stop = 1;
+        }
+      }
+      if (__shfl_sync(0xffffffffu, stop, 0)) return false;
+      __nanosleep(backoff_ns(spin));
+    }
+    st_release_u64(v.end, (static_cast<uint64_t>(seq) << 32) | h);
+    return true;
+  }
+};
+
+// Heap side: HeapCore fed from the ring.  Every call is made by all 32 lanes.
+template <int ROWS, int FIXED_K = 0>
+struct RowSink : HeapCore<ROWS, FIXED_K> {
+  using Core = HeapCore<ROWS, FIXED_K>;
+  using Core::push;
+  using Core::tau;
+  using Core::n;
+  using Core::k;
+  RingView<ROWS> v;
+  int R;
+  uint32_t t;    // records consumed
+  int tm;        // t mod R
+  uint32_t seq;  // current unit
+
+  __device__ __forceinline__ void init(uint8_t* ring_mem, int row, int R_) {
+    v.bind(ring_mem, row, R_);
+    R = R_;
+    t = 0;
+    tm = 0;
+    seq = 0;
+  }
+
+  // Start the next unit: empty heap, and a threshold word of the new unit
+  // (-inf), which also tells the filter warp that the previous end mark has
+  // been taken.
+  __device__ __forceinline__ void begin_unit(uint8_t* heap_mem, int row, int cap) {
+    ++seq;
+    Core::init_heap(heap_mem, row, cap);
+    st_release_u64(v.tauw, (static_cast<uint64_t>(seq) << 32) | __float_as_uint(-INFINITY));
+  }
+
+  // Expand records t .. lim-1 into the heap, in two phases.
+  // 1. Each lane copies the elements of its records that beat tau into its
+  //    stage (predicated stores, in key order), as many records as the stage
+  //    surely holds, then frees those ring slots.
+  // 2. The warp walks the stages in lockstep, one element per lane per step,
+  //    re-checking each against the current root.
+  // Then the new threshold is published.
+  __device__ __forceinline__ void consume(uint32_t lim) {
+    constexpr int SC = RingView<ROWS>::kStage;
+    // while the heap is filling its root says nothing: use the unit's floor
+    float thr = tau;
+    if (n < k) {
+      const uint64_t fw = ld_acquire_u64(v.flw);
+      if (static_cast<uint32_t>(fw >> 32) == seq) thr = __uint_as_float(static_cast<uint32_t>(fw));
+    }
+    int cnt = 0;
+    int s = tm;
+    uint32_t tt = t;
+    while (tt != lim && cnt + 8 <= SC) {
+      const float4 a = v.lo[s * ROWS];
+      const float4 b = v.hi[s * ROWS];
+      const uint32_t j0 = v.rj[s * ROWS];
+      const float e8[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        const bool pass = e8[e] > thr;
+        st_shared_u2_if(pass, v.stage + cnt * ROWS, __float_as_uint(e8[e]), j0 + e);
+        cnt += pass ? 1 : 0;
+      }
+      s = s + 1 == R ? 0 : s + 1;
+      ++tt;
+    }
+    tm = s;
+    t = tt;
+    st_release_u32(v.tail, t);
+    const int mx = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(cnt));
+    uint2 c = cnt > 0 ? v.stage[0] : make_uint2(0u, 0u);
+    if (FIXED_K == 64 && __all_sync(0xffffffffu, n == k)) {
+      // every heap is full: one straight-line replace per step
+      uint64_t r = Core::root;
+      for (int q = 0; q < mx; ++q) {
+        const uint2 cn = q + 1 < cnt ? v.stage[(q + 1) * ROWS] : make_uint2(0u, 0u);
+        const uint64_t key = make_key(__uint_as_float(c.x), c.y);
+        r = Core::replace_root64_pred(key, q < cnt && key > r, r);
+        c = cn;
+      }
+      Core::root = r;
+      tau = key_score(r);
     } else {
-      if (n < k && n > 1)
-        for (int p = (n - 2) / 4; p >= 0; --p) sift_down(get(p), p, n);
-      for (int m = n - 1; m > 0; --m) {
-        const uint64_t x = get(m);
-        put(m, get(0));
-        sift_down(x, 0, m);
+      for (int q = 0; q < mx; ++q) {
+        const uint2 cn = q + 1 < cnt ? v.stage[(q + 1) * ROWS] : make_uint2(0u, 0u);
+        const float x = __uint_as_float(c.x);
+        if (q < cnt && x > tau) push(make_key(x, c.y));  // tau >= thr once the heap is full
+        c = cn;
       }
+    }
+    if (n == k) st_relaxed_u64(v.tauw, (static_cast<uint64_t>(seq) << 32) | __float_as_uint(tau));
+  }
+
+  // Consume this unit's records until its end mark has been seen and every
+  // record before it expanded.  A batch starts when some row has `batch`
+  // records pending (larger batches keep more lanes busy in the lockstep
+  // expansion) or when the unit's records are all in.  `batch` must not
+  // exceed the free-slot margin the filter waits for, or both would wait.
+  // Returns false if the CTA aborts or nothing happens within the wait limit.
+  __device__ __forceinline__ bool drain_unit(int batch, const DevCtl& ctl, volatile int* abort_flag) {
+    unsigned long long t0 = 0;
+    uint32_t idle = 0;
+    for (;;) {
+      // head before end: a head that already counts records of the next
+      // unit implies that this unit's end mark is visible
+      const uint32_t hd = ld_acquire_u32(v.head);
+      const uint64_t e = ld_acquire_u64(v.end);
+      const bool fin = static_cast<uint32_t>(e >> 32) == seq;
+      const uint32_t lim = fin ? static_cast<uint32_t>(e) : hd;
+      const int pend = static_cast<int>(lim - t);
+      const bool all_fin = __all_sync(0xffffffffu, fin);
+      if (__any_sync(0xffffffffu, pend >= batch) || (all_fin && __any_sync(0xffffffffu, pend != 0))) {
+        consume(lim);
+        idle = 0;
+        continue;
+      }
+      if (all_fin) return true;
+      int stop = 0;
+      if ((threadIdx.x & 31) == 0 && (idle & 15u) == 0) {
+        if (idle == 0) {
+          t0 = global_ns();
+        } else if (*abort_flag) {
+          stop = 1;
+        } else if (global_ns() - t0 > ctl.wait_limit_ns) {
+          atomicOr(ctl.error, kDevErrTimeout);
+          *abort_flag = 1;
+          stop = 1;
+        }
+      }
+      if (__shfl_sync(0xffffffffu, stop, 0)) return false;
+      __nanosleep(backoff_ns(idle));
+      ++idle;
     }
   }
 };
@@ -347,7 +753,7 @@ __device__ __forceinline__ uint4 f32x8_to_bf16(const float (&f)[8]) {
 }
 
 // Softmax over the kept entries (Eq. 4) and the weighted sum of value rows,
-// for one row whose heap has been sorted.  Values are rows of D elements of
+// for one row, in any order of its kept entries.  Values are rows of D elements of
 // type T (float or bf16) starting at `vbase` (row j at vbase + j * D); the
 // result is written to `orow` (D elements of T).  Accumulation is fp32 over
 // 64-column slices so that at most 64 accumulators are live.
@@ -356,7 +762,8 @@ __device__ __forceinline__ void softmax_gather_store(const Sel& h, const T* __re
                                                      T* __restrict__ orow) {
   constexpr int SL = D < 64 ? D : 64;
   const int n = h.n;
-  const float m = n > 0 ? key_score(h.get(0)) : 0.0f;
+  float m = -INFINITY;  // the largest kept score, for a stable exponent
+  for (int t = 0; t < n; ++t) m = fmaxf(m, key_score(h.get(t)));
 #pragma unroll 1
   for (int c0 = 0; c0 < D; c0 += SL) {
     float acc[SL];

@@ -103,6 +103,12 @@ def attention_inputs(B, H, Lq, Lk, d, *, dtype="bf16", seed=0, dist="normal"):
         q += LOWRANK_SCALE * torch.randn(B, H, Lq, r, generator=g) @ A[None]
         k = torch.randn(B, H, Lk, d, generator=g)
         k += LOWRANK_SCALE * torch.randn(B, H, Lk, r, generator=g) @ A[None]
+    elif dist == "integer":
+        # small integers: every score is an exact integer in any precision, so
+        # scores tie often and both sides see the same ties
+        q = torch.randint(-2, 3, (B, H, Lq, d), generator=g).float()
+        k = torch.randint(-2, 3, (B, H, Lk, d), generator=g).float()
+        scale = 1.0
     else:
         raise ValueError(f"unknown distribution {dist!r}")
     v = torch.randn(B, H, Lk, d, generator=g)

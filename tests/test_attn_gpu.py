@@ -169,3 +169,50 @@ def test_memory_is_linear_in_keys():
         del dq, dk, dv, out
     d = np.diff(peaks)
     assert np.allclose(d[1:] / d[:-1], 2.0, rtol=0.02), peaks
+
+
+def _exact_selection(q, k, v, topk, causal=False, rows=None):
+    """Integer-valued scores are exact on both sides: the kept lists must be identical, in order."""
+    out, idx, score = _run(q, k, v, topk, causal=causal)
+    total = q.shape[0] * q.shape[1] * q.shape[2]
+    rows = np.arange(total) if rows is None else np.asarray(rows)
+    ref = oracle.topk_attention(q, k, v, topk, causal=causal, rows=rows)
+    assert np.array_equal(idx[rows].numpy(), ref["idx"])
+    got = score[rows].numpy().astype(np.float64)
+    assert np.array_equal(np.where(ref["idx"] >= 0, got, 0.0), np.where(ref["idx"] >= 0, ref["score"], 0.0))
+    assert np.abs(out[rows].numpy() - ref["out"]).max() <= 2e-2
+    return ref
+
+
+@pytest.mark.parametrize("d,topk,Lk", [(64, 8, 8192), (64, 64, 32768), (128, 16, 16384)])
+def test_floor_prepass_with_exact_ties(d, topk, Lk):
+    # Lk >= 512 k: the kernel first scores topk groups of >= 64 keys and uses the smallest group
+    # maximum as a floor; integer scores put many keys exactly on that floor and on the k-th score
+    q, k, v = W.attention_inputs(1, 2, 256, Lk, d, dtype="bf16", seed=400 + topk, dist="integer")
+    ref = _exact_selection(q, k, v, topk)
+    # the ties are real: many rows have the k-th and (k+1)-th scores equal
+    assert np.mean(ref["score"][:, -1] == ref["next_score"]) > 0.3
+
+
+def test_floor_prepass_causal_with_exact_ties():
+    # causal: only query tiles with at least 8x the pre-pass keys in range take the floor
+    L = 16384
+    q, k, v = W.attention_inputs(1, 1, L, L, 64, dtype="bf16", seed=410, dist="integer")
+    rows = np.concatenate([np.arange(0, 64), np.arange(8000, 8300), np.arange(L - 300, L)])
+    _exact_selection(q, k, v, 8, causal=True, rows=rows)
+
+
+def test_floor_equal_to_kth_score_keeps_lowest_indices():
+    # scores in {0, 1} with about 5% ones: every pre-pass group holds a 1, so the floor is 1, equal to
+    # the k-th score, and the kept set is the lowest-index ones (the tie rule of the total order)
+    g = torch.Generator().manual_seed(420)
+    B, H, Lq, Lk, d, topk = 1, 1, 128, 16384, 64, 16
+    q = torch.zeros(B, H, Lq, d)
+    q[..., 0] = 1.0
+    k = torch.zeros(B, H, Lk, d)
+    k[..., 0] = (torch.rand(B, H, Lk, generator=g) < 0.05).float()
+    v = torch.randn(B, H, Lk, d, generator=g)
+    q, k, v = q.bfloat16(), k.bfloat16(), v.bfloat16()
+    ref = _exact_selection(q, k, v, topk)
+    ones = torch.nonzero(k[0, 0, :, 0] == 1).flatten()[:topk].int().numpy()
+    assert np.array_equal(ref["idx"][0], ones)
