@@ -72,7 +72,10 @@ struct Layout {
   static constexpr size_t OFF_Q = 0;
   static constexpr size_t OFF_K = OFF_Q + Q_BYTES;
   static constexpr size_t OFF_SEL = OFF_K + static_cast<size_t>(S) * KST_BYTES;
-  static constexpr int NBARS = 2 * S + 7;
+  // TMEM accumulators: as many N-column buffers as fit in 512 columns, at
+  // most 4, so that the MMA warp can run ahead of a selection that stalls
+  static constexpr int NACC = 512 / N < 4 ? 512 / N : 4;
+  static constexpr int NBARS = 2 * S + 3 + 2 * NACC;
   static constexpr size_t CTRL_BYTES = 256;
   static constexpr size_t kMaxSmem = 232448;
   static constexpr size_t kFixed = 1024 + OFF_SEL + CTRL_BYTES;
@@ -80,7 +83,9 @@ struct Layout {
   // Single-warp selection: pending score groups per row, as many as fit, at
   // most 24; a selection call adds up to OW/8 groups, so fewer than OW/8 + 1
   // does not work (0).  Split selection: record ring slots per row, at most
-  // 24, at least two selection calls' worth.
+  // 24; the filter reserves OW/8 slots per selection call and the heap warp
+  // starts a batch at R/2 pending (rounded down), which must not exceed
+  // R - OW/8 + 1 (else both could wait): R >= 2 OW/8 - 2; at least 2 OW/8.
   static constexpr int kMinCap = SPLIT ? 2 * (OW / 8) : OW / 8 + 1;
   __host__ __device__ static constexpr size_t heap_bytes(int topk) {
     return (Heap::heap_bytes(topk) + 15) & ~size_t(15);
@@ -133,7 +138,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
   using Sel = typename L::Sel;
   constexpr int N = L::N, S = L::S, R = L::R;
   constexpr uint32_t IDESC = idesc_bf16_f32(BM, N);
-  constexpr uint32_t TMEM_COLS = 2 * N;
+  constexpr int NACC = L::NACC;
+  constexpr uint32_t TMEM_COLS = NACC * N;
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
@@ -146,9 +152,9 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
   uint64_t* empty_k = bars + S;
   uint64_t* q_full = bars + 2 * S;
   uint64_t* q_empty = bars + 2 * S + 1;
-  uint64_t* acc_full = bars + 2 * S + 2;   // [2]
-  uint64_t* acc_empty = bars + 2 * S + 4;  // [2]
-  uint64_t* drain = bars + 2 * S + 6;
+  uint64_t* acc_full = bars + 2 * S + 2;          // [NACC]
+  uint64_t* acc_empty = bars + 2 * S + 2 + NACC;  // [NACC]
+  uint64_t* drain = bars + 2 * S + 2 + 2 * NACC;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + L::NBARS);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -162,7 +168,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     }
     mbar_init(q_full, 1);
     mbar_init(q_empty, 1);
-    for (int b = 0; b < 2; ++b) {
+    for (int b = 0; b < NACC; ++b) {
       mbar_init(&acc_full[b], 1);
       mbar_init(&acc_empty[b], 4);
     }
@@ -276,8 +282,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
           ok = false;
           break;
         }
-        const int b = acc_it & 1;
-        if (!warp_wait(&acc_empty[b], ((acc_it >> 1) & 1u) ^ 1u, ctl, abort_flag)) {
+        const int b = acc_it % NACC;
+        if (!warp_wait(&acc_empty[b], ((acc_it / NACC) & 1u) ^ 1u, ctl, abort_flag)) {
           ok = false;
           break;
         }
@@ -331,8 +337,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         // keys are -inf, so a row with a short key range gets no floor)
         float F = INFINITY, gm = -INFINITY;
         for (int kt = 0; ok && kt < npre; ++kt, ++acc_it) {
-          const int b = acc_it & 1;
-          if (!warp_wait(&acc_full[b], (acc_it >> 1) & 1u, ctl, abort_flag)) {
+          const int b = acc_it % NACC;
+          if (!warp_wait(&acc_full[b], (acc_it / NACC) & 1u, ctl, abort_flag)) {
             ok = false;
             break;
           }
@@ -372,8 +378,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         f.set_floor(F);
       }
       for (int kt = 0; ok && kt < nk; ++kt, ++acc_it) {
-        const int b = acc_it & 1;
-        if (!warp_wait(&acc_full[b], (acc_it >> 1) & 1u, ctl, abort_flag)) {
+        const int b = acc_it % NACC;
+        if (!warp_wait(&acc_full[b], (acc_it / NACC) & 1u, ctl, abort_flag)) {
           ok = false;
           break;
         }
@@ -403,8 +409,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
             f.offer(reinterpret_cast<const float(&)[OW]>(vals[h * OW]), j0 + static_cast<uint32_t>(h * OW));
           }
           if (!ok) break;
-          f.publish();
         }
+        f.publish();  // once per key tile
       }
       if (ok && !f.end_unit(ctl, abort_flag)) ok = false;
     }
@@ -449,8 +455,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
       const uint32_t lim = static_cast<uint32_t>(causal ? min(i_row + 1, Lk) : Lk);
       const int lim_min = causal ? min(qt * BM + 1, Lk) : Lk;
       for (int kt = 0; kt < nk; ++kt, ++acc_it) {
-        const int b = acc_it & 1;
-        if (!warp_wait(&acc_full[b], (acc_it >> 1) & 1u, ctl, abort_flag)) {
+        const int b = acc_it % NACC;
+        if (!warp_wait(&acc_full[b], (acc_it / NACC) & 1u, ctl, abort_flag)) {
           ok = false;
           break;
         }

@@ -162,7 +162,7 @@ struct HeapCore {
   // always read and the stores are predicated, so that a warp whose lanes
   // disagree on act runs one straight-line body.  Returns the root after
   // the call (`cur`, the current root, when act is false).
-  __device__ __forceinline__ uint64_t replace_root64_pred(uint64_t x, bool act, uint64_t cur) {
+  __device__ __forceinline__ uint64_t replace_pred(uint64_t x, bool act, uint64_t cur) {
     uint64_t ch[8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) ch[q] = get(1 + q);
@@ -659,13 +659,15 @@ struct RowSink : HeapCore<ROWS, FIXED_K> {
     st_release_u32(v.tail, t);
     const int mx = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(cnt));
     uint2 c = cnt > 0 ? v.stage[0] : make_uint2(0u, 0u);
-    if (FIXED_K == 64 && __all_sync(0xffffffffu, n == k)) {
-      // every heap is full: one straight-line replace per step
+    bool fast = false;
+    if constexpr (FIXED_K == 64) fast = __all_sync(0xffffffffu, n == k);
+    if (fast) {
+      // every kept set is full: one straight-line replace per step
       uint64_t r = Core::root;
       for (int q = 0; q < mx; ++q) {
         const uint2 cn = q + 1 < cnt ? v.stage[(q + 1) * ROWS] : make_uint2(0u, 0u);
         const uint64_t key = make_key(__uint_as_float(c.x), c.y);
-        r = Core::replace_root64_pred(key, q < cnt && key > r, r);
+        r = Core::replace_pred(key, q < cnt && key > r, r);
         c = cn;
       }
       Core::root = r;
