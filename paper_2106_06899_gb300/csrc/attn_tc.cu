@@ -386,30 +386,54 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         tc_fence_after();
         const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(b * N);
         const uint32_t jt = static_cast<uint32_t>(kt * N);
-#pragma unroll 1
-        for (int c = 0; c < N / 64; ++c) {
-          float vals[64];
-          f.refresh_tau();
+        f.refresh_tau();
+        if constexpr (N == 128) {
+          // both 64-column halves into separate registers up front: the
+          // second load never waits for the first half's record stores
+          float va[64], vb[64];
           __syncwarp();
-          tmem_ld64(taddr + c * 64, vals);
+          tmem_ld64(taddr, va);
+          tmem_ld64(taddr + 64, vb);
           tmem_wait_ld();
-          if (c == N / 64 - 1) {
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&acc_empty[b]);
-          }
-          const uint32_t j0 = jt + static_cast<uint32_t>(c * 64);
-          if (static_cast<int>(j0) + 64 > lim_min) mask_scores(vals, j0, lim);
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[b]);
+          if (static_cast<int>(jt) + 64 > lim_min) mask_scores(va, jt, lim);
+          if (static_cast<int>(jt) + 128 > lim_min) mask_scores(vb, jt + 64u, lim);
 #pragma unroll
-          for (int h = 0; h < 64 / OW; ++h) {
+          for (int h = 0; h < 4 && ok; ++h) {
             if (!f.reserve(OW / 8, ctl, abort_flag)) {
               ok = false;
               break;
             }
-            f.offer(reinterpret_cast<const float(&)[OW]>(vals[h * OW]), j0 + static_cast<uint32_t>(h * OW));
+            const float* src = h < 2 ? va + h * OW : vb + (h - 2) * OW;
+            f.offer(*reinterpret_cast<const float(*)[OW]>(src), jt + static_cast<uint32_t>(h * OW));
           }
-          if (!ok) break;
+        } else {
+#pragma unroll 1
+          for (int c = 0; c < N / 64 && ok; ++c) {
+            float vals[64];
+            __syncwarp();
+            tmem_ld64(taddr + c * 64, vals);
+            tmem_wait_ld();
+            if (c == N / 64 - 1) {
+              tc_fence_before();
+              __syncwarp();
+              if (lane == 0) mbar_arrive(&acc_empty[b]);
+            }
+            const uint32_t j0 = jt + static_cast<uint32_t>(c * 64);
+            if (static_cast<int>(j0) + 64 > lim_min) mask_scores(vals, j0, lim);
+#pragma unroll
+            for (int h = 0; h < 64 / OW; ++h) {
+              if (!f.reserve(OW / 8, ctl, abort_flag)) {
+                ok = false;
+                break;
+              }
+              f.offer(reinterpret_cast<const float(&)[OW]>(vals[h * OW]), j0 + static_cast<uint32_t>(h * OW));
+            }
+          }
         }
+        if (!ok) break;
         f.publish();  // once per key tile
       }
       if (ok && !f.end_unit(ctl, abort_flag)) ok = false;

@@ -113,20 +113,6 @@ __device__ __forceinline__ uint64_t ld_acquire_u64(const uint64_t* p) {
 }
 
 // Predicated shared-memory stores (no branch, no write when p is false).
-__device__ __forceinline__ void st_shared_f4_if(bool p, float4* dst, float a, float b, float c, float d) {
-  asm volatile(
-      "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t"
-      "@q st.shared.v4.f32 [%1], {%2, %3, %4, %5};\n\t}" ::"r"(static_cast<int>(p)),
-      "r"(smem_u32(dst)), "f"(a), "f"(b), "f"(c), "f"(d));
-}
-
-__device__ __forceinline__ void st_shared_u32_if(bool p, uint32_t* dst, uint32_t v) {
-  asm volatile(
-      "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t"
-      "@q st.shared.u32 [%1], %2;\n\t}" ::"r"(static_cast<int>(p)),
-      "r"(smem_u32(dst)), "r"(v));
-}
-
 __device__ __forceinline__ void st_shared_u2_if(bool p, uint2* dst, uint32_t a, uint32_t b) {
   asm volatile(
       "{\n\t.reg .pred q;\n\tsetp.ne.b32 q, %0, 0;\n\t"

@@ -185,6 +185,34 @@ struct HeapCore {
     return act ? top : cur;
   }
 
+  // replace_pred with the root's 8 children (slots 1..8) kept in registers
+  // by the caller across calls: level 0 needs no shared-memory round trip,
+  // and the register copy is updated with selects.  The shared-memory heap
+  // is kept identical.
+  __device__ __forceinline__ uint64_t replace_pred_rc(uint64_t x, bool act, uint64_t cur, uint64_t (&ch0)[8]) {
+    uint64_t a0;
+    int i0;
+    argmin8(ch0, a0, i0);
+    const int c0 = 1 + i0;
+    const bool go0 = act && a0 < x;
+    const int c1b = 8 * c0 + 1;
+    uint64_t ch[8];
+#pragma unroll
+    for (int q = 0; q < 8; ++q) ch[q] = get(c1b + q);
+    uint64_t a1;
+    int i1;
+    argmin8(ch, a1, i1);
+    const bool go1 = go0 && a1 < x;
+    const uint64_t top = go0 ? a0 : x;
+    const uint64_t mid = go1 ? a1 : x;
+    st_shared_u64_if(act, base, top);
+    st_shared_u64_if(go0, base + c0 * ROWS, mid);
+    st_shared_u64_if(go1, base + (c1b + i1) * ROWS, x);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) ch0[q] = (go0 && q == i0) ? mid : ch0[q];
+    return act ? top : cur;
+  }
+
   // Smallest of 8 keys and its position (tree of depth 3).
   __device__ __forceinline__ static void argmin8(const uint64_t (&ch)[8], uint64_t& m, int& i) {
     uint64_t m2[4];
@@ -529,7 +557,7 @@ struct RowFilter {
   }
 
   // Offer W scores with key indices j0 .. j0+W-1; needs W/8 free slots.
-  // A group that does not pass costs no shared-memory store (predicated).
+  // A group that does not pass costs no shared-memory store.
   template <int W>
   __device__ __forceinline__ void offer(const float (&x)[W], uint32_t j0) {
     constexpr int G = W / 8;
@@ -541,9 +569,11 @@ struct RowFilter {
 #pragma unroll
     for (int g = 0; g < G; ++g) {
       const bool pass = m[g] > tau;
-      st_shared_f4_if(pass, v.lo + hm * ROWS, x[8 * g], x[8 * g + 1], x[8 * g + 2], x[8 * g + 3]);
-      st_shared_f4_if(pass, v.hi + hm * ROWS, x[8 * g + 4], x[8 * g + 5], x[8 * g + 6], x[8 * g + 7]);
-      st_shared_u32_if(pass, v.rj + hm * ROWS, j0 + 8 * g);
+      if (pass) {  // compiled to predicated stores
+        v.lo[hm * ROWS] = make_float4(x[8 * g], x[8 * g + 1], x[8 * g + 2], x[8 * g + 3]);
+        v.hi[hm * ROWS] = make_float4(x[8 * g + 4], x[8 * g + 5], x[8 * g + 6], x[8 * g + 7]);
+        v.rj[hm * ROWS] = j0 + 8 * g;
+      }
       const int nx = hm + (pass ? 1 : 0);
       hm = nx == R ? 0 : nx;
       h += pass ? 1u : 0u;
@@ -664,10 +694,13 @@ struct RowSink : HeapCore<ROWS, FIXED_K> {
     if (fast) {
       // every kept set is full: one straight-line replace per step
       uint64_t r = Core::root;
+      uint64_t ch0[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) ch0[q] = Core::get(1 + q);
       for (int q = 0; q < mx; ++q) {
         const uint2 cn = q + 1 < cnt ? v.stage[(q + 1) * ROWS] : make_uint2(0u, 0u);
         const uint64_t key = make_key(__uint_as_float(c.x), c.y);
-        r = Core::replace_pred(key, q < cnt && key > r, r);
+        r = Core::replace_pred_rc(key, q < cnt && key > r, r, ch0);
         c = cn;
       }
       Core::root = r;
