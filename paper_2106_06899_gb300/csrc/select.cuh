@@ -185,10 +185,10 @@ struct HeapCore {
     return act ? top : cur;
   }
 
-  // replace_pred with the root's 8 children (slots 1..8) kept in registers
-  // by the caller across calls: level 0 needs no shared-memory round trip,
-  // and the register copy is updated with selects.  The shared-memory heap
-  // is kept identical.
+  // replace_pred with the root (cur) and its 8 children (slots 1..8) kept
+  // in registers by the caller across calls: level 0 needs no shared-memory
+  // round trip, and only the leaf level is written to shared memory here.
+  // The caller writes the root and ch0 back to slots 0..8 afterwards.
   __device__ __forceinline__ uint64_t replace_pred_rc(uint64_t x, bool act, uint64_t cur, uint64_t (&ch0)[8]) {
     uint64_t a0;
     int i0;
@@ -205,8 +205,6 @@ struct HeapCore {
     const bool go1 = go0 && a1 < x;
     const uint64_t top = go0 ? a0 : x;
     const uint64_t mid = go1 ? a1 : x;
-    st_shared_u64_if(act, base, top);
-    st_shared_u64_if(go0, base + c0 * ROWS, mid);
     st_shared_u64_if(go1, base + (c1b + i1) * ROWS, x);
 #pragma unroll
     for (int q = 0; q < 8; ++q) ch0[q] = (go0 && q == i0) ? mid : ch0[q];
@@ -703,6 +701,9 @@ struct RowSink : HeapCore<ROWS, FIXED_K> {
         r = Core::replace_pred_rc(key, q < cnt && key > r, r, ch0);
         c = cn;
       }
+      Core::put(0, r);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) Core::put(1 + q, ch0[q]);
       Core::root = r;
       tau = key_score(r);
     } else {
