@@ -48,7 +48,7 @@ struct TcShape;
 template <bool SPLIT>
 struct TcShape<64, SPLIT> {
   static constexpr int N = SPLIT ? 128 : 256;
-  static constexpr int S = SPLIT ? 3 : 2;
+  static constexpr int S = 2;
   static constexpr int OW = 32;
 };
 template <bool SPLIT>
@@ -84,9 +84,10 @@ struct Layout {
   // most 24; a selection call adds up to OW/8 groups, so fewer than OW/8 + 1
   // does not work (0).  Split selection: record ring slots per row, at most
   // 24; the filter reserves OW/8 slots per selection call and the heap warp
-  // starts a batch at R/2 pending (rounded down), which must not exceed
-  // R - OW/8 + 1 (else both could wait): R >= 2 OW/8 - 2; at least 2 OW/8.
+  // starts a batch at 2R/3 pending (rounded down), which must not exceed
+  // R - OW/8 + 1 (else both could wait): R >= 3 (OW/8 - 1); at least 2 OW/8.
   static constexpr int kMinCap = SPLIT ? 2 * (OW / 8) : OW / 8 + 1;
+  static_assert(!SPLIT || 2 * kMinCap / 3 <= kMinCap - OW / 8 + 1, "batch threshold above the filter margin");
   __host__ __device__ static constexpr size_t heap_bytes(int topk) {
     return (Heap::heap_bytes(topk) + 15) & ~size_t(15);
   }
@@ -449,9 +450,10 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
       decode(u, bh, qt);
       const int i_row = qt * BM + row;
       heap.begin_unit(sel_mem, row, topk);
-      // batch threshold: half the ring, below the filter's margin of OW/8
-      // free slots, so that the filter never waits on a heap warp that waits
-      if (!heap.drain_unit(rec_cap / 2, ctl, abort_flag)) break;
+      // batch threshold: two thirds of the ring, within the filter's margin
+      // of OW/8 free slots, so that the filter never waits on a heap warp
+      // that waits
+      if (!heap.drain_unit(rec_cap * 2 / 3, ctl, abort_flag)) break;
       if (i_row < Lq) {
         const size_t orow = static_cast<size_t>(bh) * Lq + i_row;
         // the softmax needs no order; only the index/score outputs are sorted

@@ -459,7 +459,7 @@ struct RowHeap : HeapCore<ROWS, FIXED_K> {
 // ignored.
 template <int ROWS>
 struct RingView {
-  static constexpr int kStage = 24;
+  static constexpr int kStage = 16;
   uint64_t* end;
   uint64_t* tauw;
   uint32_t* head;
