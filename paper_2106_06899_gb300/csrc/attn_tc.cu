@@ -133,8 +133,8 @@ template <int D, int FK, bool SPLIT>
 __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmk,
                    const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ out, int BH, int Lq, int Lk,
-                   int topk, int rec_cap, int causal, int n_units, int pre_keys, int pre_group,
-                   int32_t* __restrict__ idx, float* __restrict__ score, DevCtl ctl) {
+                   int topk, int rec_cap, int causal, int n_units, int32_t* __restrict__ idx,
+                   float* __restrict__ score, DevCtl ctl) {
   using L = Layout<D, FK, SPLIT>;
   using Sel = typename L::Sel;
   constexpr int N = L::N, S = L::S, R = L::R;
@@ -201,15 +201,6 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     const int kend = causal ? min(Lk, (qt + 1) * BM) : Lk;
     return (kend + N - 1) / N;
   };
-  // Floor pre-pass (split variant): the first pre_keys keys are scored once
-  // more ahead of the unit, in topk groups of pre_group keys; the smallest
-  // group maximum is a floor of the row's k-th largest score.  Only where it
-  // costs at most an eighth of the unit's keys.
-  auto pre_tiles = [&](int qt) {
-    if (pre_group == 0) return 0;
-    const int kend = causal ? min(Lk, (qt + 1) * BM) : Lk;
-    return kend / 8 >= pre_keys ? (pre_keys + N - 1) / N : 0;
-  };
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -231,10 +222,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         for (int r = 0; r < R; ++r) tma_load_3d(q_s + r * BM * 128, &tmq, q_full, r * 64, qt * BM, bh);
       }
       ++q_issued;
-      const int npre = pre_tiles(qt);
-      const int nk = npre + key_tiles(qt);
-      for (int t = 0; t < nk; ++t) {
-        const int kt = t < npre ? t : t - npre;
+      const int nk = key_tiles(qt);
+      for (int kt = 0; kt < nk; ++kt) {
         const int s = it % S;
         const uint32_t ph = (it / S) & 1u;
         if (!warp_wait(&empty_k[s], ph ^ 1u, ctl, abort_flag)) {
@@ -276,7 +265,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         break;
       }
       tc_fence_after();
-      const int nk = pre_tiles(qt) + key_tiles(qt);
+      const int nk = key_tiles(qt);
       for (int kt = 0; kt < nk; ++kt, ++it, ++acc_it) {
         const int s = it % S;
         if (!warp_wait(&full_k[s], (it / S) & 1u, ctl, abort_flag)) {
@@ -330,54 +319,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
       f.begin_unit();
       const int i_row = qt * BM + row;
       const int nk = key_tiles(qt);
-      const int npre = pre_tiles(qt);
       const uint32_t lim = static_cast<uint32_t>(causal ? min(i_row + 1, Lk) : Lk);
       const int lim_min = causal ? min(qt * BM + 1, Lk) : Lk;
-      if (npre > 0) {
-        // pre-pass: F = min over the topk groups of their maxima (masked
-        // keys are -inf, so a row with a short key range gets no floor)
-        float F = INFINITY, gm = -INFINITY;
-        for (int kt = 0; ok && kt < npre; ++kt, ++acc_it) {
-          const int b = acc_it % NACC;
-          if (!warp_wait(&acc_full[b], (acc_it / NACC) & 1u, ctl, abort_flag)) {
-            ok = false;
-            break;
-          }
-          tc_fence_after();
-          const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(b * N);
-#pragma unroll 1
-          for (int c = 0; c < N / 64; ++c) {
-            float vals[64];
-            __syncwarp();
-            tmem_ld64(taddr + c * 64, vals);
-            tmem_wait_ld();
-            if (c == N / 64 - 1) {
-              tc_fence_before();
-              __syncwarp();
-              if (lane == 0) mbar_arrive(&acc_empty[b]);
-            }
-            const uint32_t j0 = static_cast<uint32_t>(kt * N + c * 64);
-            if (static_cast<int>(j0) + 64 > lim_min) mask_scores(vals, j0, lim);
-#pragma unroll
-            for (int h = 0; h < 2; ++h) {
-              const uint32_t jh = j0 + 32u * h;
-              if (jh < static_cast<uint32_t>(pre_keys)) {
-                float hm = vals[32 * h];
-#pragma unroll
-                for (int e = 1; e < 31; e += 2) hm = max3f(hm, vals[32 * h + e], vals[32 * h + e + 1]);
-                hm = fmaxf(hm, vals[32 * h + 31]);
-                gm = fmaxf(gm, hm);
-                if (((jh + 32u) & static_cast<uint32_t>(pre_group - 1)) == 0u) {
-                  F = fminf(F, gm);
-                  gm = -INFINITY;
-                }
-              }
-            }
-          }
-        }
-        if (!ok) break;
-        f.set_floor(F);
-      }
       for (int kt = 0; ok && kt < nk; ++kt, ++acc_it) {
         const int b = acc_it % NACC;
         if (!warp_wait(&acc_full[b], (acc_it / NACC) & 1u, ctl, abort_flag)) {
@@ -545,18 +488,9 @@ int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t 
       cudaSuccess)
     return -1;
   const int grid = n_units < num_sms ? n_units : num_sms;
-  // floor pre-pass (split only): topk groups of the largest power of two
-  // >= 64 keys such that the pre-pass reads at most Lk / 8 keys
-  int pre_keys = 0, pre_group = 0;
-  if (SPLIT)
-    for (long long gs = 64; static_cast<long long>(a.topk) * gs * 8 <= a.Lk; gs *= 2) {
-      pre_group = static_cast<int>(gs);
-      pre_keys = static_cast<int>(a.topk * gs);
-    }
   kern<<<grid, kThreads<SPLIT>, smem, st>>>(tmq, tmk, static_cast<const __nv_bfloat16*>(a.v),
                                             static_cast<__nv_bfloat16*>(a.out), BH, a.Lq, a.Lk, a.topk,
-                                            L::cap(a.topk), a.causal, n_units, pre_keys, pre_group, a.idx,
-                                            a.score, ctl);
+                                            L::cap(a.topk), a.causal, n_units, a.idx, a.score, ctl);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 

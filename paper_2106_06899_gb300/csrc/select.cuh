@@ -41,17 +41,6 @@ __device__ __forceinline__ float key_score(uint64_t key) { return unord_f32(stat
 
 __device__ __forceinline__ uint32_t key_index(uint64_t key) { return ~static_cast<uint32_t>(key); }
 
-// The largest float below s (s itself if it is -inf): x > below_f32(s)
-// exactly when x >= s, for any float x that is not NaN.  -0 is skipped: it
-// compares equal to +0, so the float below +0 is the negative denormal of
-// least magnitude.
-__device__ __forceinline__ float below_f32(float s) {
-  if (s == -INFINITY) return s;
-  uint32_t o = ord_f32(s) - 1u;
-  if (o == 0x7FFFFFFFu) o -= 1u;
-  return unord_f32(o);
-}
-
 // The heap of one row: a min-heap of its k best packed keys in shared memory
 // ([slot][row] layout, ROWS rows per slot).  push() offers one key; sort()
 // turns the heap into the kept keys in selection order.  The 4-ary layout
@@ -447,8 +436,6 @@ struct RowHeap : HeapCore<ROWS, FIXED_K> {
 //   tauw  u64  (unit sequence number << 32) | bits of the heap root's score
 //   head  u32  records written (filter, release store)
 //   tail  u32  records consumed (heap warp, release store)
-//   flw   u64  (unit sequence number << 32) | bits of a score floor that the
-//              filter found before its first record (a pre-pass), or 0
 //   R record slots, then kStage (score, index) pairs: the heap warp's own
 //   list of the elements it is about to offer to the heap.  The heap warp
 //   copies the qualifying elements out of the records first and frees the
@@ -464,13 +451,12 @@ struct RingView {
   uint64_t* tauw;
   uint32_t* head;
   uint32_t* tail;
-  uint64_t* flw;
   float4* lo;
   float4* hi;
   uint32_t* rj;
   uint2* stage;
 
-  __host__ __device__ static constexpr size_t ctl_bytes() { return static_cast<size_t>(ROWS) * 32; }
+  __host__ __device__ static constexpr size_t ctl_bytes() { return static_cast<size_t>(ROWS) * 24; }
   __host__ __device__ static constexpr size_t bytes(int R) {
     return ctl_bytes() + static_cast<size_t>(ROWS) * (static_cast<size_t>(R) * 36 + kStage * 8);
   }
@@ -481,7 +467,6 @@ struct RingView {
     tauw = reinterpret_cast<uint64_t*>(mem + ROWS * 8) + row;
     head = reinterpret_cast<uint32_t*>(mem + ROWS * 16) + row;
     tail = reinterpret_cast<uint32_t*>(mem + ROWS * 20) + row;
-    flw = reinterpret_cast<uint64_t*>(mem + ROWS * 24) + row;
     uint8_t* r = mem + ctl_bytes();
     const size_t nrec = static_cast<size_t>(R);
     lo = reinterpret_cast<float4*>(r) + row;
@@ -578,16 +563,6 @@ struct RowFilter {
     }
   }
 
-  // Adopt a floor F of the row's k-th largest score (at least k scores of
-  // the row are >= F): from now on only scores >= F pass, and the heap warp
-  // applies the same floor while its heap is filling.  Called before the
-  // unit's first record.
-  __device__ __forceinline__ void set_floor(float F) {
-    const float below = below_f32(F);  // x > below  <=>  x >= F
-    tau = fmaxf(tau, below);
-    st_release_u64(v.flw, (static_cast<uint64_t>(seq) << 32) | __float_as_uint(below));
-  }
-
   // Make the records written so far visible to the heap warp.
   __device__ __forceinline__ void publish() { st_release_u32(v.head, h); }
 
@@ -659,12 +634,7 @@ struct RowSink : HeapCore<ROWS, FIXED_K> {
   // Then the new threshold is published.
   __device__ __forceinline__ void consume(uint32_t lim) {
     constexpr int SC = RingView<ROWS>::kStage;
-    // while the heap is filling its root says nothing: use the unit's floor
-    float thr = tau;
-    if (n < k) {
-      const uint64_t fw = ld_acquire_u64(v.flw);
-      if (static_cast<uint32_t>(fw >> 32) == seq) thr = __uint_as_float(static_cast<uint32_t>(fw));
-    }
+    const float thr = tau;  // -inf while the heap is filling
     int cnt = 0;
     int s = tm;
     uint32_t tt = t;
@@ -710,7 +680,7 @@ struct RowSink : HeapCore<ROWS, FIXED_K> {
       for (int q = 0; q < mx; ++q) {
         const uint2 cn = q + 1 < cnt ? v.stage[(q + 1) * ROWS] : make_uint2(0u, 0u);
         const float x = __uint_as_float(c.x);
-        if (q < cnt && x > tau) push(make_key(x, c.y));  // tau >= thr once the heap is full
+        if (q < cnt && x > tau) push(make_key(x, c.y));
         c = cn;
       }
     }

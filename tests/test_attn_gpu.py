@@ -185,26 +185,26 @@ def _exact_selection(q, k, v, topk, causal=False, rows=None):
 
 
 @pytest.mark.parametrize("d,topk,Lk", [(64, 8, 8192), (64, 64, 32768), (128, 16, 16384)])
-def test_floor_prepass_with_exact_ties(d, topk, Lk):
-    # Lk >= 512 k: the kernel first scores topk groups of >= 64 keys and uses the smallest group
-    # maximum as a floor; integer scores put many keys exactly on that floor and on the k-th score
+def test_exact_ties_long_rows(d, topk, Lk):
+    # integer scores: many keys share the k-th score, so the kept set depends on the lower-index
+    # rule alone; the split kernel's filter, ring and heap must reproduce it exactly
     q, k, v = W.attention_inputs(1, 2, 256, Lk, d, dtype="bf16", seed=400 + topk, dist="integer")
     ref = _exact_selection(q, k, v, topk)
     # the ties are real: many rows have the k-th and (k+1)-th scores equal
     assert np.mean(ref["score"][:, -1] == ref["next_score"]) > 0.3
 
 
-def test_floor_prepass_causal_with_exact_ties():
-    # causal: only query tiles with at least 8x the pre-pass keys in range take the floor
+def test_exact_ties_causal():
+    # causal rows of every length, integer scores: exact kept lists, including rows i < k
     L = 16384
     q, k, v = W.attention_inputs(1, 1, L, L, 64, dtype="bf16", seed=410, dist="integer")
     rows = np.concatenate([np.arange(0, 64), np.arange(8000, 8300), np.arange(L - 300, L)])
     _exact_selection(q, k, v, 8, causal=True, rows=rows)
 
 
-def test_floor_equal_to_kth_score_keeps_lowest_indices():
-    # scores in {0, 1} with about 5% ones: every pre-pass group holds a 1, so the floor is 1, equal to
-    # the k-th score, and the kept set is the lowest-index ones (the tie rule of the total order)
+def test_binary_scores_keep_lowest_indices():
+    # scores in {0, 1} with about 5% ones: the k-th score is 1 and is shared by hundreds of keys, so
+    # the kept set is the lowest-index ones (the tie rule of the total order)
     g = torch.Generator().manual_seed(420)
     B, H, Lq, Lk, d, topk = 1, 1, 128, 16384, 64, 16
     q = torch.zeros(B, H, Lq, d)
