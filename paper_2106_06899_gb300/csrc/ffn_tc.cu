@@ -18,9 +18,10 @@
 //    Rows also share L across slices through one word per row (the k-th
 //    largest of any subset of keys is <= that of all keys).
 // 2. ffn_finalize_kernel (one CTA per token).  Reads the row's candidates
-//    from every slice, keeps the exact top-k by the total order (score
-//    descending, index ascending) with a bitonic sort in shared memory,
-//    applies ReLU and gathers the W2 rows with fp32 accumulation.
+//    from every slice and keeps the exact top-k by the total order (score
+//    descending, index ascending), sorted, in the workspace.
+// 3. ffn_gather_kernel (one CTA per column chunk and token, chunk-major).
+//    Applies ReLU and gathers the W2 rows with fp32 accumulation.
 //
 // No [tokens x d_ff] score matrix is ever written to device memory.
 #include <algorithm>
@@ -52,7 +53,7 @@ constexpr int kFinalMaxCand = 8192;  // candidates at or above the final bound h
 
 struct Plan {
   int n_rt, tiles, n_sl, n_units, cap;
-  size_t off_cnt, off_tau, bytes;
+  size_t off_cnt, off_tau, off_kept, bytes;
 };
 
 Plan make_plan(int N, int d_model, int d_ff, int topk, int num_sms) {
@@ -87,7 +88,8 @@ Plan make_plan(int N, int d_model, int d_ff, int topk, int num_sms) {
   const size_t rows_sl = static_cast<size_t>(N) * p.n_sl;
   p.off_cnt = rows_sl * p.cap * sizeof(uint2);
   p.off_tau = p.off_cnt + rows_sl * sizeof(int);
-  p.bytes = p.off_tau + static_cast<size_t>(N) * sizeof(uint32_t);
+  p.off_kept = (p.off_tau + static_cast<size_t>(N) * sizeof(uint32_t) + 15) & ~size_t(15);
+  p.bytes = p.off_kept + static_cast<size_t>(N) * topk * sizeof(uint64_t);  // kept keys per token
   return p;
 }
 
@@ -465,7 +467,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
 }
 
-// One CTA per token row: exact top-k among its candidates, ReLU, W2 gather.
+// One CTA per token row: exact top-k among its candidates.
 //
 // Only candidates >= L (the row's shared bound) can be in the top-k.  An
 // MSB-first radix select over their ordered score keys (11, 11 and 10 bits;
@@ -495,10 +497,9 @@ __device__ __forceinline__ int warp_append(int* counter, bool take) {
 }
 
 __global__ void __launch_bounds__(kFinalThreads)
-    ffn_finalize_kernel(const __nv_bfloat16* __restrict__ W2, float* __restrict__ out, int d_model, int topk,
-                        int n_sl, int cap, const uint2* __restrict__ cand, const int* __restrict__ cand_cnt,
-                        const uint32_t* __restrict__ row_tau, int32_t* __restrict__ idx,
-                        float* __restrict__ score, DevCtl ctl) {
+    ffn_finalize_kernel(uint64_t* __restrict__ kept, int topk, int n_sl, int cap, const uint2* __restrict__ cand,
+                        const int* __restrict__ cand_cnt, const uint32_t* __restrict__ row_tau,
+                        int32_t* __restrict__ idx, float* __restrict__ score, DevCtl ctl) {
   extern __shared__ uint64_t keys[];  // [kFinalMaxCand]; the first kHistBins words double as the histogram
   __shared__ uint32_t csum[kFinalThreads];
   __shared__ int n_keys, n_ties, bad, sh_digit, sh_above;
@@ -700,40 +701,8 @@ __global__ void __launch_bounds__(kFinalThreads)
     }
   }
   }
-  // ReLU over the kept scores and the weighted sum of W2 rows (fp32), eight
-  // rows in flight per thread
-  float* orow = out + static_cast<size_t>(row) * d_model;
-  for (int c0 = tid * 4; c0 < d_model; c0 += kFinalThreads * 4) {
-    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
-    int t = 0;
-    for (; t + 8 <= topk; t += 8) {
-      uint2 raw[8];
-      float w[8];
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const uint64_t key = keys[t + u];
-        w[u] = fmaxf(key_score(key), 0.0f);
-        raw[u] = __ldg(reinterpret_cast<const uint2*>(W2 + static_cast<size_t>(key_index(key)) * d_model + c0));
-      }
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        a0 = fmaf(w[u], __uint_as_float(raw[u].x << 16), a0);
-        a1 = fmaf(w[u], __uint_as_float(raw[u].x & 0xFFFF0000u), a1);
-        a2 = fmaf(w[u], __uint_as_float(raw[u].y << 16), a2);
-        a3 = fmaf(w[u], __uint_as_float(raw[u].y & 0xFFFF0000u), a3);
-      }
-    }
-    for (; t < topk; ++t) {
-      const uint64_t key = keys[t];
-      const float w = fmaxf(key_score(key), 0.0f);
-      const uint2 raw = __ldg(reinterpret_cast<const uint2*>(W2 + static_cast<size_t>(key_index(key)) * d_model + c0));
-      a0 = fmaf(w, __uint_as_float(raw.x << 16), a0);
-      a1 = fmaf(w, __uint_as_float(raw.x & 0xFFFF0000u), a1);
-      a2 = fmaf(w, __uint_as_float(raw.y << 16), a2);
-      a3 = fmaf(w, __uint_as_float(raw.y & 0xFFFF0000u), a3);
-    }
-    *reinterpret_cast<float4*>(orow + c0) = make_float4(a0, a1, a2, a3);
-  }
+  // the kept keys, in selection order, for the gather kernel
+  for (int t = tid; t < topk; t += kFinalThreads) kept[static_cast<size_t>(row) * topk + t] = keys[t];
   if (idx || score) {
     for (int t = tid; t < topk; t += kFinalThreads) {
       const uint64_t key = keys[t];
@@ -741,6 +710,57 @@ __global__ void __launch_bounds__(kFinalThreads)
       if (score) score[static_cast<size_t>(row) * topk + t] = key_score(key);
     }
   }
+}
+
+// ReLU over the kept scores and the weighted sum of the matching W2 rows
+// (fp32).  One CTA per (column chunk, token), chunk-major: all tokens read
+// their rows' first kGatherCols columns before any reads the next chunk, so
+// that the W2 columns being read (d_ff x kGatherCols bf16, 32 MB at d_ff =
+// 65536) stay resident in L2 while every token visits them.  Each thread
+// owns 4 columns and keeps 8 rows in flight.
+constexpr int kGatherCols = 256;
+constexpr int kGatherThreads = kGatherCols / 4;
+
+__global__ void __launch_bounds__(kGatherThreads)
+    ffn_gather_kernel(const __nv_bfloat16* __restrict__ W2, float* __restrict__ out, int N, int d_model, int topk,
+                      const uint64_t* __restrict__ kept) {
+  extern __shared__ uint64_t gkeys[];  // [topk]
+  const int row = blockIdx.x % N;
+  const int chunk = blockIdx.x / N;
+  const int tid = threadIdx.x;
+  for (int t = tid; t < topk; t += kGatherThreads) gkeys[t] = kept[static_cast<size_t>(row) * topk + t];
+  __syncthreads();
+  const int c0 = chunk * kGatherCols + tid * 4;
+  if (c0 >= d_model) return;
+  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  int t = 0;
+  for (; t + 8 <= topk; t += 8) {
+    uint2 raw[8];
+    float w[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const uint64_t key = gkeys[t + u];
+      w[u] = fmaxf(key_score(key), 0.0f);
+      raw[u] = __ldg(reinterpret_cast<const uint2*>(W2 + static_cast<size_t>(key_index(key)) * d_model + c0));
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      a0 = fmaf(w[u], __uint_as_float(raw[u].x << 16), a0);
+      a1 = fmaf(w[u], __uint_as_float(raw[u].x & 0xFFFF0000u), a1);
+      a2 = fmaf(w[u], __uint_as_float(raw[u].y << 16), a2);
+      a3 = fmaf(w[u], __uint_as_float(raw[u].y & 0xFFFF0000u), a3);
+    }
+  }
+  for (; t < topk; ++t) {
+    const uint64_t key = gkeys[t];
+    const float w = fmaxf(key_score(key), 0.0f);
+    const uint2 raw = __ldg(reinterpret_cast<const uint2*>(W2 + static_cast<size_t>(key_index(key)) * d_model + c0));
+    a0 = fmaf(w, __uint_as_float(raw.x << 16), a0);
+    a1 = fmaf(w, __uint_as_float(raw.x & 0xFFFF0000u), a1);
+    a2 = fmaf(w, __uint_as_float(raw.y << 16), a2);
+    a3 = fmaf(w, __uint_as_float(raw.y & 0xFFFF0000u), a3);
+  }
+  *reinterpret_cast<float4*>(out + static_cast<size_t>(row) * d_model + c0) = make_float4(a0, a1, a2, a3);
 }
 
 bool make_tmap_bf16_2d(CUtensorMap* map, const void* base, uint64_t dim0, uint64_t dim1, uint32_t box1) {
@@ -792,10 +812,15 @@ int ffn_tc(const FfnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
   if (cudaFuncSetAttribute(ffn_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(kFinalSmem)) != cudaSuccess)
     return -1;
-  ffn_finalize_kernel<<<a.N, kFinalThreads, kFinalSmem, st>>>(static_cast<const __nv_bfloat16*>(a.W2), a.out, a.d_model,
-                                                      a.topk, p.n_sl, p.cap, cand, cnt, tau, a.idx, a.score, ctl);
+  uint64_t* kept = reinterpret_cast<uint64_t*>(ws + p.off_kept);
+  ffn_finalize_kernel<<<a.N, kFinalThreads, kFinalSmem, st>>>(kept, a.topk, p.n_sl, p.cap, cand, cnt, tau, a.idx,
+                                                              a.score, ctl);
   if (cudaGetLastError() != cudaSuccess) return -1;
-  return 2;
+  const int n_chunks = (a.d_model + kGatherCols - 1) / kGatherCols;
+  ffn_gather_kernel<<<n_chunks * a.N, kGatherThreads, static_cast<size_t>(a.topk) * sizeof(uint64_t), st>>>(
+      static_cast<const __nv_bfloat16*>(a.W2), a.out, a.N, a.d_model, a.topk, kept);
+  if (cudaGetLastError() != cudaSuccess) return -1;
+  return 3;
 }
 
 }  // namespace topk
