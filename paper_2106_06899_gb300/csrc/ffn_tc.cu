@@ -3,7 +3,7 @@
 //
 // Keys and values are the rows of W1 and W2 (Sec. 2.1), so a token x_i keeps
 // the k largest scores s_ij = x_i . W1_j over all d_ff keys, applies ReLU to
-// them and sums the matching rows of W2.  Two kernels:
+// them and sums the matching rows of W2.  Three kernels:
 //
 // 1. ffn_score_select_kernel (persistent, one CTA per SM).  A work unit is a
 //    128-token tile x one slice of the d_ff keys.  TMA streams x and W1
