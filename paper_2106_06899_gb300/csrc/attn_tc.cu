@@ -494,12 +494,16 @@ int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t 
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
-// Split selection where its heaps and rings fit; the 8-ary heap for k = 64.
+// Split selection where its heaps and rings fit, else the single-warp kernel.
 template <int D>
 int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
+  // fixed heap shapes: 8-ary for k = 64, two-level (8 x 16) for 65 <= k <= 137
+  const bool two_level = a.topk >= 65 && a.topk <= 137;
   if (a.topk == 64 && Layout<D, 64, true>::fits(64)) return launch_tc_k<D, 64, true>(a, ctl, num_sms, st);
+  if (two_level && Layout<D, 128, true>::fits(a.topk)) return launch_tc_k<D, 128, true>(a, ctl, num_sms, st);
   if (Layout<D, 0, true>::fits(a.topk)) return launch_tc_k<D, 0, true>(a, ctl, num_sms, st);
   if (a.topk == 64 && Layout<D, 64, false>::fits(64)) return launch_tc_k<D, 64, false>(a, ctl, num_sms, st);
+  if (two_level && Layout<D, 128, false>::fits(a.topk)) return launch_tc_k<D, 128, false>(a, ctl, num_sms, st);
   return launch_tc_k<D, 0, false>(a, ctl, num_sms, st);
 }
 

@@ -51,7 +51,28 @@ struct HeapCore {
   // FIXED_K == 64: an 8-ary heap of exactly 64 keys, padded with 9 sentinel
   // slots (largest key) so that every interior node has 8 children: a root
   // replacement is two fully unrolled levels of 8 independent loads.
+  // FIXED_K == 128: a two-level heap of any k in [65, 137] keys (k is a
+  // runtime value): the root (slot 0), 8 nodes (slots 1..8) and up to 16
+  // leaves under node c (slots 9 + 16 (c - 1) .. + 15 that are below k; a
+  // missing leaf reads as the largest key).  A root replacement is 8 + 16
+  // independent loads, without sentinel slots.
   static constexpr int kPad = FIXED_K == 64 ? 9 : 0;
+  static constexpr int kLeaves = FIXED_K == 128 ? 16 : 8;  // children per level-1 node (fixed shapes)
+
+  // slot of the q-th child of level-1 node c (1..8) in the fixed shapes
+  __device__ __forceinline__ static int leaf_slot(int c, int q) {
+    if constexpr (FIXED_K == 128)
+      return 9 + 16 * (c - 1) + q;
+    else
+      return 8 * c + 1 + q;
+  }
+  // key at a leaf slot (the largest key where the two-level shape has none)
+  __device__ __forceinline__ uint64_t leaf_key(int s) const {
+    if constexpr (FIXED_K == 128)
+      return s < k ? get(s) : ~0ull;
+    else
+      return get(s);
+  }
   uint64_t* base;  // &heap[slot 0][this row]
   int k;           // capacity
   int n;           // entries filled
@@ -184,20 +205,72 @@ struct HeapCore {
     argmin8(ch0, a0, i0);
     const int c0 = 1 + i0;
     const bool go0 = act && a0 < x;
-    const int c1b = 8 * c0 + 1;
-    uint64_t ch[8];
+    uint64_t ch[kLeaves];
 #pragma unroll
-    for (int q = 0; q < 8; ++q) ch[q] = get(c1b + q);
+    for (int q = 0; q < kLeaves; ++q) ch[q] = leaf_key(leaf_slot(c0, q));
     uint64_t a1;
     int i1;
-    argmin8(ch, a1, i1);
+    argmin_n(ch, a1, i1);
     const bool go1 = go0 && a1 < x;
     const uint64_t top = go0 ? a0 : x;
     const uint64_t mid = go1 ? a1 : x;
-    st_shared_u64_if(go1, base + (c1b + i1) * ROWS, x);
+    st_shared_u64_if(go1, base + leaf_slot(c0, i1) * ROWS, x);
 #pragma unroll
     for (int q = 0; q < 8; ++q) ch0[q] = (go0 && q == i0) ? mid : ch0[q];
     return act ? top : cur;
+  }
+
+  // Smallest of NC keys (a power of two) and its first position (a tree).
+  template <int NC>
+  __device__ __forceinline__ static void argmin_n(const uint64_t (&ch)[NC], uint64_t& m, int& i) {
+    uint64_t v[NC];
+    int p[NC];
+#pragma unroll
+    for (int q = 0; q < NC; ++q) {
+      v[q] = ch[q];
+      p[q] = q;
+    }
+#pragma unroll
+    for (int w = NC / 2; w >= 1; w /= 2) {
+#pragma unroll
+      for (int q = 0; q < w; ++q) {
+        const bool lo = v[q] <= v[q + w];
+        v[q] = lo ? v[q] : v[q + w];
+        p[q] = lo ? p[q] : p[q + w];
+      }
+    }
+    m = v[0];
+    i = p[0];
+  }
+
+  // Sift x down from slot p in the two-level shape of k keys.
+  __device__ __forceinline__ void sift128(uint64_t x, int p) {
+    for (;;) {
+      int first, cnt;
+      if (p == 0) {
+        first = 1;
+        cnt = 8;
+      } else if (p <= 8) {
+        first = 9 + 16 * (p - 1);
+        cnt = k - first < 16 ? k - first : 16;
+        if (cnt <= 0) break;
+      } else {
+        break;
+      }
+      uint64_t a = get(first);
+      int ca = first;
+      for (int q = first + 1; q < first + cnt; ++q) {
+        const uint64_t b = get(q);
+        if (b < a) {
+          a = b;
+          ca = q;
+        }
+      }
+      if (a >= x) break;
+      put(p, a);
+      p = ca;
+    }
+    put(p, x);
   }
 
   // Smallest of 8 keys and its position (tree of depth 3).
@@ -229,6 +302,8 @@ struct HeapCore {
           // build the 8-ary heap: nodes 8..1 (level 1), then the root
           for (int p = 8; p >= 1; --p) sift_down8(get(p), p);
           sift_down8(get(0), 0);
+        } else if constexpr (FIXED_K == 128) {
+          for (int p = 8; p >= 0; --p) sift128(get(p), p);
         } else {
           for (int p = (k - 2) / 4; p >= 0; --p) sift_down(get(p), p, k);
         }
@@ -238,6 +313,9 @@ struct HeapCore {
     } else if (x > root) {
       if constexpr (FIXED_K == 64) {
         root = replace_root64(x);
+      } else if constexpr (FIXED_K == 128) {
+        sift128(x, 0);
+        root = get(0);
       } else {
         sift_down(x, 0, k);
         root = get(0);
@@ -282,7 +360,8 @@ struct HeapCore {
         sift_down8(x, 0, m);
       }
     } else {
-      if (n < k && n > 1)
+      // the 4-ary order; the fixed 128 shape is not one, so it is rebuilt
+      if ((n < k || FIXED_K == 128) && n > 1)
         for (int p = (n - 2) / 4; p >= 0; --p) sift_down(get(p), p, n);
       for (int m = n - 1; m > 0; --m) {
         const uint64_t x = get(m);
@@ -373,13 +452,38 @@ struct RowHeap : HeapCore<ROWS, FIXED_K> {
     float x = -INFINITY;
     uint32_t j = 0;
     if (cnt > 0) fetch(0, x, j);
-    for (int t = 0; t < mx; ++t) {
-      float xn = -INFINITY;
-      uint32_t jn = 0;
-      if (t + 1 < cnt) fetch(t + 1, xn, jn);
-      if (t < cnt && x > tau) push(make_key(x, j));
-      x = xn;
-      j = jn;
+    bool fast = false;
+    if constexpr (FIXED_K == 64 || FIXED_K == 128) fast = __all_sync(0xffffffffu, Core::n == Core::k);
+    if (fast) {
+      // every heap is full: one straight-line replace per step, the root and
+      // its 8 children in registers, written back once
+      uint64_t r = Core::root;
+      uint64_t ch0[8];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) ch0[q] = Core::get(1 + q);
+      for (int t = 0; t < mx; ++t) {
+        float xn = -INFINITY;
+        uint32_t jn = 0;
+        if (t + 1 < cnt) fetch(t + 1, xn, jn);
+        const uint64_t key = make_key(x, j);
+        r = Core::replace_pred_rc(key, t < cnt && key > r, r, ch0);
+        x = xn;
+        j = jn;
+      }
+      Core::put(0, r);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) Core::put(1 + q, ch0[q]);
+      Core::root = r;
+      tau = key_score(r);
+    } else {
+      for (int t = 0; t < mx; ++t) {
+        float xn = -INFINITY;
+        uint32_t jn = 0;
+        if (t + 1 < cnt) fetch(t + 1, xn, jn);
+        if (t < cnt && x > tau) push(make_key(x, j));
+        x = xn;
+        j = jn;
+      }
     }
     rc = 0;
   }
@@ -658,7 +762,7 @@ struct RowSink : HeapCore<ROWS, FIXED_K> {
     const int mx = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(cnt));
     uint2 c = cnt > 0 ? v.stage[0] : make_uint2(0u, 0u);
     bool fast = false;
-    if constexpr (FIXED_K == 64) fast = __all_sync(0xffffffffu, n == k);
+    if constexpr (FIXED_K == 64 || FIXED_K == 128) fast = __all_sync(0xffffffffu, n == k);
     if (fast) {
       // every kept set is full: one straight-line replace per step
       uint64_t r = Core::root;

@@ -216,3 +216,17 @@ def test_binary_scores_keep_lowest_indices():
     ref = _exact_selection(q, k, v, topk)
     ones = torch.nonzero(k[0, 0, :, 0] == 1).flatten()[:topk].int().numpy()
     assert np.array_equal(ref["idx"][0], ones)
+
+
+@pytest.mark.parametrize("d", [64, 128])
+@pytest.mark.parametrize("topk", [65, 96, 112, 137])
+def test_two_level_heap_sizes(d, topk):
+    # 65 <= k <= 137 keep their set in the fixed two-level heap (8 nodes, up to 16 leaves each,
+    # missing leaves read as the largest key); ragged lengths, several query tiles per head
+    q, k, v = W.attention_inputs(1, 2, 300, 1500, d, dtype="bf16", seed=500 + topk + d)
+    _check(q, k, v, topk, "bf16")
+
+
+def test_two_level_heap_exact_ties():
+    q, k, v = W.attention_inputs(1, 2, 256, 8192, 64, dtype="bf16", seed=510, dist="integer")
+    _exact_selection(q, k, v, 100)
