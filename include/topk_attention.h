@@ -33,10 +33,14 @@
  *     enqueue work and return without synchronising.
  *   - Every argument is validated before anything is launched, so an error
  *     return never leaves a partial write.
- *   - Scratch, where a call needs it, is taken from the stream-ordered
- *     allocator on `stream` and released on it; its size is reported by the
+ *   - Scratch, where a call needs it, is taken on `stream` from a
+ *     stream-ordered memory pool that the library owns (one per device) and
+ *     returned to it on `stream`; its size is reported by the
  *     *_workspace_bytes queries and is linear in the number of query rows,
- *     never proportional to Lq * Lk.
+ *     never proportional to Lq * Lk.  The pool keeps returned memory
+ *     reserved for later calls (up to the largest amount in use at once)
+ *     until the process exits, so that repeated calls do not map device
+ *     memory again each time.
  *
  * Return codes: 0 on success, else one of the negative TOPK_ERR_* values;
  * topk_error_string() describes them.
@@ -147,9 +151,18 @@ size_t topk_ffn_workspace_bytes(int N, int d_model, int d_ff, int topk);
 
 /*
  * End-to-end variants taking HOST pointers (pinned memory is fastest).  They
- * stage the inputs into stream-ordered device memory, run the call above on
- * `stream`, copy the result back and synchronise `stream` before returning.
- * Sizes and dtypes as above.
+ * stage the inputs into device memory from the library's pool, run the call
+ * above on `stream`, copy the result back and synchronise `stream` before
+ * returning.  Sizes and dtypes as above.
+ *   - topk_attn_fwd_host splits the B*H heads into up to 8 consecutive
+ *     slices when there are enough query tiles (about 12 per SM per slice)
+ *     and launches one call per slice on `stream`; each slice's inputs are
+ *     copied on a copy stream of the library and its output copied back on
+ *     another, so the copies of neighbouring slices overlap the kernels.
+ *     The result is identical to one call over all heads.
+ *   - topk_ffn_fwd_host copies x and W1 first and W2 on a copy stream while
+ *     the score and selection kernels run; the W2 gather waits for it.
+ *   The copy streams are shared by all host-buffer calls on a device.
  */
 int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq,
                        int Lk, int d, int topk, int chunk, int causal, int dtype, void* stream);

@@ -59,6 +59,46 @@ DevCtl make_ctl(DeviceState* s) {
   return c;
 }
 
+// Device memory the library allocates itself (feed-forward scratch, the
+// staging buffers of the host-buffer calls) comes from one stream-ordered
+// pool per device that keeps freed memory reserved for the next call, so a
+// steady stream of calls of one shape maps device memory once instead of on
+// every call.  Two non-blocking streams per device carry the host-buffer
+// calls' copies, so that they overlap the kernels on the caller's stream.
+struct HostPipe {
+  std::once_flag once;
+  cudaMemPool_t pool = nullptr;
+  cudaStream_t h2d = nullptr, d2h = nullptr;
+  bool ok = false;
+};
+HostPipe g_pipe[kMaxDevices];
+
+HostPipe* host_pipe() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+  HostPipe& s = g_pipe[dev];
+  std::call_once(s.once, [&s, dev]() {
+    cudaMemPoolProps props;
+    std::memset(&props, 0, sizeof props);
+    props.allocType = cudaMemAllocationTypePinned;
+    props.handleTypes = cudaMemHandleTypeNone;
+    props.location.type = cudaMemLocationTypeDevice;
+    props.location.id = dev;
+    if (cudaMemPoolCreate(&s.pool, &props) != cudaSuccess) return;
+    cuuint64_t keep = ~0ull;  // never hand freed memory back between calls
+    if (cudaMemPoolSetAttribute(s.pool, cudaMemPoolAttrReleaseThreshold, &keep) != cudaSuccess) return;
+    if (cudaStreamCreateWithFlags(&s.h2d, cudaStreamNonBlocking) != cudaSuccess) return;
+    if (cudaStreamCreateWithFlags(&s.d2h, cudaStreamNonBlocking) != cudaSuccess) return;
+    s.ok = true;
+  });
+  return s.ok ? &s : nullptr;
+}
+
+bool pool_alloc(void** p, size_t bytes, cudaStream_t st) {
+  HostPipe* hp = host_pipe();
+  return hp && cudaMallocFromPoolAsync(p, bytes, hp->pool, st) == cudaSuccess;
+}
+
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 int validate_attn(const AttnArgs& a) {
@@ -111,9 +151,7 @@ int run_ffn(FfnArgs a, cudaStream_t st) {
   const DevCtl ctl = make_ctl(dev);
   const size_t ws = ffn_workspace_bytes(a.N, a.d_model, a.d_ff, a.topk);
   void* buf = nullptr;
-  if (ws) {
-    if (cudaMallocAsync(&buf, ws, st) != cudaSuccess) return TOPK_ERR_CUDA;
-  }
+  if (ws && !pool_alloc(&buf, ws, st)) return TOPK_ERR_CUDA;
   a.workspace = buf;
   a.workspace_bytes = ws;
   int n = ffn_tc(a, ctl, dev->num_sms, st);
@@ -216,6 +254,10 @@ int host_call_status(int rc) {
 }
 }  // namespace
 
+// Head slices of a host-buffer attention call: enough 128-query tiles per
+// slice for about 12 per SM (little tail in each launch), at most 8 slices.
+constexpr int kHostSlicesMax = 8;
+
 int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk, int d,
                        int topk, int chunk, int causal, int dtype, void* stream) {
   if (!q || !k || !v || !out) return TOPK_ERR_INVALID_ARG;
@@ -224,28 +266,80 @@ int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, i
                reinterpret_cast<void*>(16), B, H, Lq, Lk, d, topk, chunk, causal, dtype, nullptr, nullptr};
   int rc = validate_attn(chk);
   if (rc) return rc;
+  DeviceState* dev = device_state();
+  HostPipe* hp = host_pipe();
+  if (!dev || !hp) return TOPK_ERR_NO_DEVICE;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const size_t eb = elem_bytes(dtype);
-  const size_t qb = static_cast<size_t>(B) * H * Lq * d * eb, kb = static_cast<size_t>(B) * H * Lk * d * eb;
+  const int BH = B * H;
+  const size_t qh = static_cast<size_t>(Lq) * d * eb, kh = static_cast<size_t>(Lk) * d * eb;
+  const long long tiles = static_cast<long long>(BH) * ((Lq + 127) / 128);
+  int P = static_cast<int>(tiles / (12LL * dev->num_sms));
+  P = P < 1 ? 1 : (P > BH ? BH : (P > kHostSlicesMax ? kHostSlicesMax : P));
+
   void *dq = nullptr, *dk = nullptr, *dv = nullptr, *dout = nullptr;
-  if (cudaMallocAsync(&dq, qb, st) != cudaSuccess || cudaMallocAsync(&dk, kb, st) != cudaSuccess ||
-      cudaMallocAsync(&dv, kb, st) != cudaSuccess || cudaMallocAsync(&dout, qb, st) != cudaSuccess) {
-    rc = TOPK_ERR_CUDA;
-  } else if (cudaMemcpyAsync(dq, q, qb, cudaMemcpyHostToDevice, st) != cudaSuccess ||
-             cudaMemcpyAsync(dk, k, kb, cudaMemcpyHostToDevice, st) != cudaSuccess ||
-             cudaMemcpyAsync(dv, v, kb, cudaMemcpyHostToDevice, st) != cudaSuccess) {
-    rc = TOPK_ERR_CUDA;
-  } else {
-    rc = topk_attn_fwd(dq, dk, dv, dout, B, H, Lq, Lk, d, topk, chunk, causal, dtype, stream);
-    if (rc == TOPK_OK && cudaMemcpyAsync(out, dout, qb, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+  cudaEvent_t ready = nullptr, h2d_done = nullptr, d2h_done = nullptr;
+  cudaEvent_t ev_in[kHostSlicesMax] = {}, ev_out[kHostSlicesMax] = {};
+  auto mk = [](cudaEvent_t* e) { return cudaEventCreateWithFlags(e, cudaEventDisableTiming) == cudaSuccess; };
+  bool good = pool_alloc(&dq, BH * qh, st) && pool_alloc(&dk, BH * kh, st) && pool_alloc(&dv, BH * kh, st) &&
+              pool_alloc(&dout, BH * qh, st) && mk(&ready) && mk(&h2d_done) && mk(&d2h_done);
+  for (int s = 0; good && s < P; ++s) good = mk(&ev_in[s]) && mk(&ev_out[s]);
+  // the copy streams start once the allocations on `st` are in place
+  good = good && cudaEventRecord(ready, st) == cudaSuccess && cudaStreamWaitEvent(hp->h2d, ready, 0) == cudaSuccess &&
+         cudaStreamWaitEvent(hp->d2h, ready, 0) == cudaSuccess;
+  if (!good) rc = TOPK_ERR_CUDA;
+  // slice s: its inputs on the h2d stream, its launch on `st` after them,
+  // its output on the d2h stream after the launch; the copies of slices
+  // s + 1 and s - 1 overlap the kernel of slice s
+  int launches = 0;
+  for (int s = 0; rc == TOPK_OK && s < P; ++s) {
+    const size_t h0 = static_cast<size_t>(static_cast<long long>(BH) * s / P);
+    const size_t h1 = static_cast<size_t>(static_cast<long long>(BH) * (s + 1) / P);
+    const size_t nh = h1 - h0;
+    uint8_t* sq = static_cast<uint8_t*>(dq) + h0 * qh;
+    uint8_t* sk = static_cast<uint8_t*>(dk) + h0 * kh;
+    uint8_t* sv = static_cast<uint8_t*>(dv) + h0 * kh;
+    uint8_t* so = static_cast<uint8_t*>(dout) + h0 * qh;
+    if (cudaMemcpyAsync(sq, static_cast<const uint8_t*>(q) + h0 * qh, nh * qh, cudaMemcpyHostToDevice, hp->h2d) !=
+            cudaSuccess ||
+        cudaMemcpyAsync(sk, static_cast<const uint8_t*>(k) + h0 * kh, nh * kh, cudaMemcpyHostToDevice, hp->h2d) !=
+            cudaSuccess ||
+        cudaMemcpyAsync(sv, static_cast<const uint8_t*>(v) + h0 * kh, nh * kh, cudaMemcpyHostToDevice, hp->h2d) !=
+            cudaSuccess ||
+        cudaEventRecord(ev_in[s], hp->h2d) != cudaSuccess || cudaStreamWaitEvent(st, ev_in[s], 0) != cudaSuccess) {
       rc = TOPK_ERR_CUDA;
+      break;
+    }
+    rc = topk_attn_fwd(sq, sk, sv, so, 1, static_cast<int>(nh), Lq, Lk, d, topk, chunk, causal, dtype, stream);
+    if (rc != TOPK_OK) break;
+    launches += t_last_launches;
+    if (cudaEventRecord(ev_out[s], st) != cudaSuccess || cudaStreamWaitEvent(hp->d2h, ev_out[s], 0) != cudaSuccess ||
+        cudaMemcpyAsync(static_cast<uint8_t*>(out) + h0 * qh, so, nh * qh, cudaMemcpyDeviceToHost, hp->d2h) !=
+            cudaSuccess) {
+      rc = TOPK_ERR_CUDA;
+      break;
+    }
   }
-  const int launches = t_last_launches;
+  // the buffers go back to the pool on `st` only after both copy streams
+  // are done with everything enqueued above
+  if (!(h2d_done && d2h_done && cudaEventRecord(h2d_done, hp->h2d) == cudaSuccess &&
+        cudaEventRecord(d2h_done, hp->d2h) == cudaSuccess && cudaStreamWaitEvent(st, h2d_done, 0) == cudaSuccess &&
+        cudaStreamWaitEvent(st, d2h_done, 0) == cudaSuccess)) {
+    cudaStreamSynchronize(hp->h2d);
+    cudaStreamSynchronize(hp->d2h);
+    if (rc == TOPK_OK) rc = TOPK_ERR_CUDA;
+  }
   if (dq) cudaFreeAsync(dq, st);
   if (dk) cudaFreeAsync(dk, st);
   if (dv) cudaFreeAsync(dv, st);
   if (dout) cudaFreeAsync(dout, st);
   if (cudaStreamSynchronize(st) != cudaSuccess && rc == TOPK_OK) rc = TOPK_ERR_CUDA;
+  for (cudaEvent_t e : {ready, h2d_done, d2h_done})
+    if (e) cudaEventDestroy(e);
+  for (int s = 0; s < P; ++s) {
+    if (ev_in[s]) cudaEventDestroy(ev_in[s]);
+    if (ev_out[s]) cudaEventDestroy(ev_out[s]);
+  }
   t_last_launches = launches;
   return host_call_status(rc);
 }
@@ -257,28 +351,47 @@ int topk_ffn_fwd_host(const void* x, const void* W1, const void* W2, void* out, 
               reinterpret_cast<float*>(16), N, d_model, d_ff, topk, nullptr, nullptr, nullptr, 0};
   int rc = validate_ffn(chk);
   if (rc) return rc;
+  HostPipe* hp = host_pipe();
+  if (!hp) return TOPK_ERR_NO_DEVICE;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   const size_t xb = static_cast<size_t>(N) * d_model * 2, wb = static_cast<size_t>(d_ff) * d_model * 2;
   const size_t ob = static_cast<size_t>(N) * d_model * 4;
   void *dx = nullptr, *d1 = nullptr, *d2 = nullptr, *dout = nullptr;
-  if (cudaMallocAsync(&dx, xb, st) != cudaSuccess || cudaMallocAsync(&d1, wb, st) != cudaSuccess ||
-      cudaMallocAsync(&d2, wb, st) != cudaSuccess || cudaMallocAsync(&dout, ob, st) != cudaSuccess) {
-    rc = TOPK_ERR_CUDA;
-  } else if (cudaMemcpyAsync(dx, x, xb, cudaMemcpyHostToDevice, st) != cudaSuccess ||
-             cudaMemcpyAsync(d1, W1, wb, cudaMemcpyHostToDevice, st) != cudaSuccess ||
-             cudaMemcpyAsync(d2, W2, wb, cudaMemcpyHostToDevice, st) != cudaSuccess) {
+  cudaEvent_t ready = nullptr, in_ready = nullptr, w2_ready = nullptr, h2d_done = nullptr;
+  auto mk = [](cudaEvent_t* e) { return cudaEventCreateWithFlags(e, cudaEventDisableTiming) == cudaSuccess; };
+  bool good = pool_alloc(&dx, xb, st) && pool_alloc(&d1, wb, st) && pool_alloc(&d2, wb, st) &&
+              pool_alloc(&dout, ob, st) && mk(&ready) && mk(&in_ready) && mk(&w2_ready) && mk(&h2d_done);
+  // x and W1 first (the score kernel needs them), then W2, which only the
+  // last kernel (the gather) reads: its copy overlaps the first two kernels
+  good = good && cudaEventRecord(ready, st) == cudaSuccess && cudaStreamWaitEvent(hp->h2d, ready, 0) == cudaSuccess &&
+         cudaMemcpyAsync(dx, x, xb, cudaMemcpyHostToDevice, hp->h2d) == cudaSuccess &&
+         cudaMemcpyAsync(d1, W1, wb, cudaMemcpyHostToDevice, hp->h2d) == cudaSuccess &&
+         cudaEventRecord(in_ready, hp->h2d) == cudaSuccess &&
+         cudaMemcpyAsync(d2, W2, wb, cudaMemcpyHostToDevice, hp->h2d) == cudaSuccess &&
+         cudaEventRecord(w2_ready, hp->h2d) == cudaSuccess && cudaStreamWaitEvent(st, in_ready, 0) == cudaSuccess;
+  if (!good) {
     rc = TOPK_ERR_CUDA;
   } else {
-    rc = topk_ffn_fwd(dx, d1, d2, dout, N, d_model, d_ff, topk, stream);
+    FfnArgs a{dx, d1, d2, static_cast<float*>(dout), N, d_model, d_ff, topk, nullptr, nullptr, nullptr, 0};
+    a.w2_ready = w2_ready;
+    rc = run_ffn(a, st);
     if (rc == TOPK_OK && cudaMemcpyAsync(out, dout, ob, cudaMemcpyDeviceToHost, st) != cudaSuccess)
       rc = TOPK_ERR_CUDA;
   }
   const int launches = t_last_launches;
+  // every copy enqueued on the h2d stream ends before the buffers are freed
+  if (!(h2d_done && cudaEventRecord(h2d_done, hp->h2d) == cudaSuccess &&
+        cudaStreamWaitEvent(st, h2d_done, 0) == cudaSuccess)) {
+    cudaStreamSynchronize(hp->h2d);
+    if (rc == TOPK_OK) rc = TOPK_ERR_CUDA;
+  }
   if (dx) cudaFreeAsync(dx, st);
   if (d1) cudaFreeAsync(d1, st);
   if (d2) cudaFreeAsync(d2, st);
   if (dout) cudaFreeAsync(dout, st);
   if (cudaStreamSynchronize(st) != cudaSuccess && rc == TOPK_OK) rc = TOPK_ERR_CUDA;
+  for (cudaEvent_t e : {ready, in_ready, w2_ready, h2d_done})
+    if (e) cudaEventDestroy(e);
   t_last_launches = launches;
   return host_call_status(rc);
 }

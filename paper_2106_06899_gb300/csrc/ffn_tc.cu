@@ -817,6 +817,7 @@ int ffn_tc(const FfnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
                                                               a.score, ctl);
   if (cudaGetLastError() != cudaSuccess) return -1;
   const int n_chunks = (a.d_model + kGatherCols - 1) / kGatherCols;
+  if (a.w2_ready && cudaStreamWaitEvent(st, a.w2_ready, 0) != cudaSuccess) return -1;
   ffn_gather_kernel<<<n_chunks * a.N, kGatherThreads, static_cast<size_t>(a.topk) * sizeof(uint64_t), st>>>(
       static_cast<const __nv_bfloat16*>(a.W2), a.out, a.N, a.d_model, a.topk, kept);
   if (cudaGetLastError() != cudaSuccess) return -1;

@@ -37,6 +37,9 @@ struct FfnArgs {
   float* score;
   void* workspace;
   size_t workspace_bytes;
+  // if set, the W2 gather (the last kernel) waits for this event first: the
+  // host-buffer entry copies W2 while the earlier kernels run
+  cudaEvent_t w2_ready = nullptr;
 };
 
 // Each launcher returns the number of kernel launches (> 0) on success,

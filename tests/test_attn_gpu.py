@@ -148,6 +148,18 @@ def test_e2e_host_entry_matches_device_entry():
     assert torch.equal(host_out, dev)
 
 
+@pytest.mark.parametrize("B,H,L,causal", [(3, 5, 32768, False), (2, 32, 8192, True)])
+def test_e2e_host_entry_in_head_slices_matches_device_entry(B, H, L, causal):
+    # enough query tiles that the host-buffer call splits the heads into slices
+    # (uneven for 15 heads) whose copies overlap the other slices' kernels
+    q, k, v = W.attention_inputs(B, H, L, L, 64, dtype="bf16", seed=17)
+    dev = T.attention(q.cuda(), k.cuda(), v.cuda(), 64, 1024, causal).cpu()
+    host_out = torch.empty_like(q).pin_memory()
+    T.topk_attn_fwd_host(q.pin_memory(), k.pin_memory(), v.pin_memory(), host_out, 64, 1024, causal)
+    assert T.topk_last_launch_count() >= 2
+    assert torch.equal(host_out, dev)
+
+
 def test_memory_is_linear_in_keys():
     # Sec. 2.2: memory O(C L_K) for a fixed chunk; here the kernel holds no per-call device scratch at
     # all, so the peak is the inputs and outputs themselves, linear in L_K
