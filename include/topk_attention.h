@@ -155,7 +155,7 @@ size_t topk_ffn_workspace_bytes(int N, int d_model, int d_ff, int topk);
  * above on `stream`, copy the result back and synchronise `stream` before
  * returning.  Sizes and dtypes as above.
  *   - topk_attn_fwd_host splits the B*H heads into up to 8 consecutive
- *     slices when there are enough query tiles (about 12 per SM per slice)
+ *     slices when there are enough query tiles (about 6 per SM per slice)
  *     and launches one call per slice on `stream`; each slice's inputs are
  *     copied on a copy stream of the library and its output copied back on
  *     another, so the copies of neighbouring slices overlap the kernels.

@@ -254,8 +254,11 @@ int host_call_status(int rc) {
 }
 }  // namespace
 
-// Head slices of a host-buffer attention call: enough 128-query tiles per
-// slice for about 12 per SM (little tail in each launch), at most 8 slices.
+// Head slices of a host-buffer attention call: about 6 or more 128-query
+// tiles per SM in each slice (the persistent launch of a slice then loses
+// little to its last, partial wave), at most 8 slices.  More slices expose
+// less copy time at the two ends (the first slice's inputs, the last
+// slice's output).
 constexpr int kHostSlicesMax = 8;
 
 int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk, int d,
@@ -274,7 +277,7 @@ int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, i
   const int BH = B * H;
   const size_t qh = static_cast<size_t>(Lq) * d * eb, kh = static_cast<size_t>(Lk) * d * eb;
   const long long tiles = static_cast<long long>(BH) * ((Lq + 127) / 128);
-  int P = static_cast<int>(tiles / (12LL * dev->num_sms));
+  int P = static_cast<int>(tiles / (6LL * dev->num_sms));
   P = P < 1 ? 1 : (P > BH ? BH : (P > kHostSlicesMax ? kHostSlicesMax : P));
 
   void *dq = nullptr, *dk = nullptr, *dv = nullptr, *dout = nullptr;
