@@ -50,6 +50,7 @@ constexpr size_t SMEM_A = 1024 + OFF_CTRL + 256;
 
 constexpr int kFinalThreads = 256;
 constexpr int kFinalMaxCand = 8192;  // candidates at or above the final bound held in shared memory
+constexpr int kFinalVec = 4;         // 16-byte candidate vectors each finalize thread loads per step
 
 struct Plan {
   int n_rt, tiles, n_sl, n_units, cap;
@@ -523,20 +524,33 @@ __global__ void __launch_bounds__(kFinalThreads)
     if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
     return;
   }
-  // visit every candidate slot of the row; all threads iterate together
+  // visit every candidate slot of the row; all threads iterate together.
+  // Each thread loads kFinalVec 16-byte vectors (two candidates each) before
+  // it visits any of them, so that many loads are in flight per thread (the
+  // lists are read from device memory).  A list starts on a 16-byte
+  // boundary and has an even capacity, so a vector never leaves its list;
+  // entries at or past the count are skipped.
   auto for_each = [&](auto&& f) {
     for (int sl = 0; sl < n_sl; ++sl) {
       const int c = cand_cnt[static_cast<size_t>(row) * n_sl + sl];
-      const uint2* lst = cand + (static_cast<size_t>(row) * n_sl + sl) * cap;
-      for (int b0 = 0; b0 < c; b0 += kFinalThreads) {
-        const int i = b0 + tid;
-        uint2 e = make_uint2(0u, 0u);
-        bool valid = i < c;
-        if (valid) {
-          e = lst[i];
-          valid = __uint_as_float(e.x) >= L;
+      const uint4* lst = reinterpret_cast<const uint4*>(cand + (static_cast<size_t>(row) * n_sl + sl) * cap);
+      for (int b0 = 0; b0 < c; b0 += 2 * kFinalVec * kFinalThreads) {
+        uint4 w[kFinalVec];
+#pragma unroll
+        for (int u = 0; u < kFinalVec; ++u) {
+          const int i = b0 + 2 * (u * kFinalThreads + tid);
+          w[u] = i < c ? lst[i / 2] : make_uint4(0u, 0u, 0u, 0u);
         }
-        f(valid, valid ? ord_f32(__uint_as_float(e.x)) : 0u, e.y);
+#pragma unroll
+        for (int u = 0; u < kFinalVec; ++u) {
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {
+            const int i = b0 + 2 * (u * kFinalThreads + tid) + h;
+            const uint32_t sx = h ? w[u].z : w[u].x, jx = h ? w[u].w : w[u].y;
+            const bool valid = i < c && __uint_as_float(sx) >= L;
+            f(valid, valid ? ord_f32(__uint_as_float(sx)) : 0u, jx);
+          }
+        }
       }
     }
   };
