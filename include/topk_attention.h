@@ -36,8 +36,9 @@
  *   - Scratch, where a call needs it, is taken on `stream` from a
  *     stream-ordered memory pool that the library owns (one per device) and
  *     returned to it on `stream`; its size is reported by the
- *     *_workspace_bytes queries and is linear in the number of query rows,
- *     never proportional to Lq * Lk.  The pool keeps returned memory
+ *     *_workspace_bytes queries and is never proportional to Lq * Lk: a
+ *     fixed amount per SM for attention, linear in the tokens for the
+ *     feed-forward layer.  The pool keeps returned memory
  *     reserved for later calls (up to the largest amount in use at once)
  *     until the process exits, so that repeated calls do not map device
  *     memory again each time.
@@ -83,9 +84,11 @@ enum {
  *   topk         : 1 <= topk <= Lk; the supported maximum is 512.
  *   chunk        : query-chunk size (Sec. 2.2), >= 1; a scheduling hint only.
  *   causal       : 0 or 1.
+ *   Scratch: topk_attn_workspace_bytes() (a fixed amount per SM, or none).
  * Errors: TOPK_ERR_INVALID_ARG / TOPK_ERR_UNSUPPORTED before any launch;
- *         TOPK_ERR_CUDA if a launch fails.  Device-side timeouts surface on
- *         the next call or through topk_check().
+ *         TOPK_ERR_CUDA if a launch fails (or the scratch cannot be had).
+ *         Device-side timeouts surface on the next call or through
+ *         topk_check().
  */
 int topk_attn_fwd(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk,
                   int d, int topk, int chunk, int causal, int dtype, void* stream);
@@ -145,7 +148,13 @@ int topk_ffn_fwd_noalloc(const void* x, const void* W1, const void* W2, void* ou
                          int d_ff, int topk, void* stream);
 
 /* Bytes of stream-ordered scratch the calls above take for these arguments
- * (0 if none).  Returns 0 as well when the arguments are invalid. */
+ * (0 if none).  Returns 0 as well when the arguments are invalid.
+ *   - attention: the bf16 tensor-core kernel with split selection parks each
+ *     work unit's kept keys for its epilogue warps: per CTA (one per SM, at
+ *     most one per 128-query tile) 4 x 2 x topk x 32 keys of 8 bytes plus
+ *     256 counts of 4 bytes, whatever Lq and Lk are.  Sized for the current
+ *     device, or for 152 SMs (a GB300) when no device is visible.
+ *   - feed-forward: linear in N (see topk_ffn_fwd). */
 size_t topk_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, int topk, int chunk, int dtype);
 size_t topk_ffn_workspace_bytes(int N, int d_model, int d_ff, int topk);
 

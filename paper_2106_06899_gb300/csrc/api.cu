@@ -19,6 +19,7 @@ namespace {
 __device__ unsigned g_device_error;  // one word per device, OR of kDevErr* flags
 
 constexpr int kMaxDevices = 64;
+constexpr int kAssumedSms = 152;  // SMs of a GB300, for size queries made without a device
 struct DeviceState {
   std::once_flag once;
   unsigned* error_word = nullptr;
@@ -124,7 +125,14 @@ int run_attn(const AttnArgs& a, cudaStream_t st) {
   if (!dev) return TOPK_ERR_NO_DEVICE;
   if (dev->cc_major != 10 || dev->cc_minor != 3) return TOPK_ERR_NO_DEVICE;
   const DevCtl ctl = make_ctl(dev);
-  int n = attn_tc(a, ctl, dev->num_sms, st);
+  const size_t ws = attn_tc_workspace_bytes(a, dev->num_sms);
+  void* buf = nullptr;
+  if (ws && !pool_alloc(&buf, ws, st)) return TOPK_ERR_CUDA;
+  AttnArgs b = a;
+  b.workspace = buf;
+  b.workspace_bytes = ws;
+  int n = attn_tc(b, ctl, dev->num_sms, st);
+  if (buf) cudaFreeAsync(buf, st);
   if (n == 0) n = attn_simt(a, st);
   if (n == 0) return TOPK_ERR_UNSUPPORTED;
   if (n < 0) return TOPK_ERR_CUDA;
@@ -228,8 +236,14 @@ int topk_ffn_fwd_indices(const void* x, const void* W1, const void* W2, void* ou
 size_t topk_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, int topk, int chunk, int dtype) {
   AttnArgs a{reinterpret_cast<void*>(16), reinterpret_cast<void*>(16), reinterpret_cast<void*>(16),
              reinterpret_cast<void*>(16), B, H, Lq, Lk, d, topk, chunk, 0, dtype, nullptr, nullptr};
-  (void)validate_attn(a);
-  return 0;  // the attention kernels keep their state in shared memory and TMEM
+  if (validate_attn(a) != TOPK_OK) return 0;
+  // sized for the current device; for a GB300 (152 SMs) when none is visible
+  int num_sms = kAssumedSms;
+  int dev = 0;
+  cudaDeviceProp p;
+  if (cudaGetDevice(&dev) == cudaSuccess && cudaGetDeviceProperties(&p, dev) == cudaSuccess)
+    num_sms = p.multiProcessorCount;
+  return attn_tc_workspace_bytes(a, num_sms);
 }
 
 size_t topk_ffn_workspace_bytes(int N, int d_model, int d_ff, int topk) {

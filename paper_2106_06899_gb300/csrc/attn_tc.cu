@@ -18,9 +18,13 @@
 //               that beat the row's threshold into the row's record ring
 //   warps 6..9  heap: warp w serves the rows of warp w-4 (same TMEM lane
 //               quarter, same SM sub-partition); it expands the records into
-//               the heaps, publishes the rising threshold and, after the
-//               unit's last record, does the sort/softmax/gather epilogue
-//               while its filter warp already reads the next unit's scores.
+//               the heaps and publishes the rising threshold.  After the
+//               unit's last record it parks the kept keys in a small device
+//               buffer (two slots per warp) and starts the next unit at once,
+//               when its filter warp sends the most records.
+//   warps 10,11 epilogue: warp 10 + e takes the parked keys of the rows of
+//               lane quarters 2e and 2e+1, applies the softmax over them and
+//               gathers the matching value rows.
 //
 // The score tile never leaves TMEM/registers: no [C x Lk] matrix is written
 // to device memory (Sec. 2.2 "Query chunking": memory O(C Lk) becomes
@@ -39,7 +43,14 @@ namespace {
 
 constexpr int BM = 128;
 template <bool SPLIT>
-constexpr int kThreads = SPLIT ? 320 : 192;
+constexpr int kThreads = SPLIT ? 384 : 192;  // split: 12 warps, three per SM sub-partition
+
+// Parked kept keys of the split kernel, per CTA: 4 heap warps x 2 slots x
+// topk keys x 32 rows (8 bytes each), then the kept count of each row.
+__host__ __device__ constexpr size_t park_keys_per_cta(int topk) { return static_cast<size_t>(4) * 2 * topk * 32; }
+__host__ __device__ constexpr size_t park_bytes(int grid, int topk) {
+  return static_cast<size_t>(grid) * (park_keys_per_cta(topk) * 8 + 4 * 2 * 32 * 4);
+}
 
 template <int D, bool SPLIT>
 struct TcShape;
@@ -117,6 +128,47 @@ __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, const 
   return ok != 0;
 }
 
+// Waits (bounded; lane 0 polls) until the shared-memory counter *ctr, which
+// only grows, reaches target; every lane then reads it with acquire
+// semantics itself, so that what the releasing warp wrote before it is
+// visible to the whole warp.  False if the CTA aborts or the limit runs out.
+__device__ __forceinline__ bool wait_count(uint32_t* ctr, uint32_t target, const DevCtl& ctl,
+                                           volatile int* abort_flag) {
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0 && static_cast<int>(ld_acquire_u32(ctr) - target) < 0) {
+    const unsigned long long t0 = global_ns();
+    for (uint32_t spin = 0;; ++spin) {
+      if (static_cast<int>(ld_acquire_u32(ctr) - target) >= 0) break;
+      if ((spin & 15u) == 15u) {
+        if (*abort_flag) {
+          ok = 0;
+          break;
+        }
+        if (global_ns() - t0 > ctl.wait_limit_ns) {
+          atomicOr(ctl.error, kDevErrTimeout);
+          *abort_flag = 1;
+          ok = 0;
+          break;
+        }
+      }
+      __nanosleep(backoff_ns(spin));
+    }
+  }
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  if (ok) (void)ld_acquire_u32(ctr);
+  return ok != 0;
+}
+
+// The kept keys of one row as parked by its heap warp (every 32nd word),
+// read through L2: they were written by another warp of the CTA.
+struct ParkedKeys {
+  const uint64_t* p;
+  int n;
+  __device__ __forceinline__ uint64_t get(int t) const {
+    return __ldcg(reinterpret_cast<const unsigned long long*>(p) + static_cast<size_t>(t) * 32);
+  }
+};
+
 // Bounded wait that ignores the abort flag: used only to drain in-flight
 // asynchronous work before the CTA exits.
 __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, const DevCtl& ctl) {
@@ -134,7 +186,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmk,
                    const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ out, int BH, int Lq, int Lk,
                    int topk, int rec_cap, int causal, int n_units, int32_t* __restrict__ idx,
-                   float* __restrict__ score, DevCtl ctl) {
+                   float* __restrict__ score, uint64_t* __restrict__ park, int* __restrict__ park_n, DevCtl ctl) {
   using L = Layout<D, FK, SPLIT>;
   using Sel = typename L::Sel;
   constexpr int N = L::N, S = L::S, R = L::R;
@@ -158,6 +210,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
   uint64_t* drain = bars + 2 * S + 2 + 2 * NACC;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + L::NBARS);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  uint32_t* pk_done = tmem_slot + 2;  // [4] split: units parked by each heap warp
+  uint32_t* ep_done = tmem_slot + 6;  // [4] split: units finished by the epilogue, per lane quarter
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -175,6 +229,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     }
     mbar_init(drain, 1);
     *abort_flag = 0;
+    for (int q = 0; q < 4; ++q) pk_done[q] = ep_done[q] = 0;
     fence_mbar_init();
   }
   if constexpr (SPLIT) {  // ring counters, end marks and thresholds start at 0
@@ -382,13 +437,15 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
       }
       if (ok && !f.end_unit(ctl, abort_flag)) ok = false;
     }
-  } else if (SPLIT) {
+  } else if (SPLIT && warp < 10) {
     // ------------------------------------------------------------ heap (split)
     const int quad = warp & 3;
     const int row = quad * 32 + lane;
     RowSink<BM, FK> heap;
     heap.init(ring_mem, row, rec_cap);
-    for (int u = blockIdx.x; u < n_units; u += gridDim.x) {
+    const size_t park0 = (static_cast<size_t>(blockIdx.x) * 4 + quad) * 2;  // this warp's first slot
+    uint32_t s = 0;                                                           // units done by this warp
+    for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++s) {
       int bh, qt;
       decode(u, bh, qt);
       const int i_row = qt * BM + row;
@@ -397,15 +454,50 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
       // of OW/8 free slots, so that the filter never waits on a heap warp
       // that waits
       if (!heap.drain_unit(rec_cap * 2 / 3, ctl, abort_flag)) break;
-      if (i_row < Lq) {
+      if (i_row < Lq && (idx || score)) {  // only the index/score outputs need the order
         const size_t orow = static_cast<size_t>(bh) * Lq + i_row;
-        // the softmax needs no order; only the index/score outputs are sorted
-        if (idx || score) heap.sort();
-        softmax_gather_store<__nv_bfloat16, D>(heap, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
-        if (idx || score)
-          write_selection(heap, idx ? idx + orow * topk : nullptr, score ? score + orow * topk : nullptr);
+        heap.sort();
+        write_selection(heap, idx ? idx + orow * topk : nullptr, score ? score + orow * topk : nullptr);
       }
+      // park the kept keys in slot s % 2; it last held unit s - 2, whose
+      // epilogue must be done
+      if (s >= 2 && !wait_count(&ep_done[quad], s - 1, ctl, abort_flag)) break;
+      const size_t slot = park0 + (s & 1u);
+      uint64_t* pk = park + slot * topk * 32 + lane;
+      const int n = i_row < Lq ? heap.n : 0;
+      for (int t = 0; t < n; ++t) pk[static_cast<size_t>(t) * 32] = heap.get(t);
+      park_n[slot * 32 + lane] = n;
       __syncwarp();
+      st_release_u32(&pk_done[quad], s + 1);
+    }
+  } else if (SPLIT) {
+    // ------------------------------------------------------------ epilogue (split)
+    // Warp 10 + e finishes the rows of lane quarters 2e and 2e + 1, unit by
+    // unit: the softmax over each row's parked kept keys (any order) and the
+    // weighted sum of their value rows.
+    const int e = warp - 10;
+    uint32_t s = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x, ++s) {
+      int bh, qt;
+      decode(u, bh, qt);
+      for (int h = 0; h < 2; ++h) {
+        const int q = 2 * e + h;
+        if (!wait_count(&pk_done[q], s + 1, ctl, abort_flag)) {
+          ok = false;
+          break;
+        }
+        const int i_row = qt * BM + q * 32 + lane;
+        const size_t slot = (static_cast<size_t>(blockIdx.x) * 4 + q) * 2 + (s & 1u);
+        const int n = __ldcg(park_n + slot * 32 + lane);
+        if (i_row < Lq && n > 0) {
+          const size_t orow = static_cast<size_t>(bh) * Lq + i_row;
+          const ParkedKeys kept{park + slot * topk * 32 + lane, n};
+          softmax_gather_store<__nv_bfloat16, D>(kept, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
+        }
+        __syncwarp();
+        st_release_u32(&ep_done[q], s + 1);
+      }
     }
   } else {
     // ------------------------------------------------------------ selection
@@ -488,23 +580,47 @@ int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t 
       cudaSuccess)
     return -1;
   const int grid = n_units < num_sms ? n_units : num_sms;
+  uint64_t* park = nullptr;
+  int* park_n = nullptr;
+  if constexpr (SPLIT) {
+    if (!a.workspace || a.workspace_bytes < park_bytes(grid, a.topk)) return -1;
+    park = static_cast<uint64_t*>(a.workspace);
+    park_n = reinterpret_cast<int*>(park + static_cast<size_t>(grid) * park_keys_per_cta(a.topk));
+  }
   kern<<<grid, kThreads<SPLIT>, smem, st>>>(tmq, tmk, static_cast<const __nv_bfloat16*>(a.v),
                                             static_cast<__nv_bfloat16*>(a.out), BH, a.Lq, a.Lk, a.topk,
-                                            L::cap(a.topk), a.causal, n_units, a.idx, a.score, ctl);
+                                            L::cap(a.topk), a.causal, n_units, a.idx, a.score, park, park_n, ctl);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
-// Split selection where its heaps and rings fit, else the single-warp kernel.
+// Which kernel serves a shape: the split selection where its heaps and rings
+// fit, else the single-warp kernel; fixed heap shapes: 8-ary for k = 64,
+// two-level (8 x 16) for 65 <= k <= 137.
+enum class TcKind { Split64, Split128, Split0, Single64, Single128, Single0 };
+
+template <int D>
+TcKind pick(int topk) {
+  const bool two_level = topk >= 65 && topk <= 137;
+  if (topk == 64 && Layout<D, 64, true>::fits(64)) return TcKind::Split64;
+  if (two_level && Layout<D, 128, true>::fits(topk)) return TcKind::Split128;
+  if (Layout<D, 0, true>::fits(topk)) return TcKind::Split0;
+  if (topk == 64 && Layout<D, 64, false>::fits(64)) return TcKind::Single64;
+  if (two_level && Layout<D, 128, false>::fits(topk)) return TcKind::Single128;
+  return TcKind::Single0;
+}
+
+bool is_split(TcKind k) { return k == TcKind::Split64 || k == TcKind::Split128 || k == TcKind::Split0; }
+
 template <int D>
 int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
-  // fixed heap shapes: 8-ary for k = 64, two-level (8 x 16) for 65 <= k <= 137
-  const bool two_level = a.topk >= 65 && a.topk <= 137;
-  if (a.topk == 64 && Layout<D, 64, true>::fits(64)) return launch_tc_k<D, 64, true>(a, ctl, num_sms, st);
-  if (two_level && Layout<D, 128, true>::fits(a.topk)) return launch_tc_k<D, 128, true>(a, ctl, num_sms, st);
-  if (Layout<D, 0, true>::fits(a.topk)) return launch_tc_k<D, 0, true>(a, ctl, num_sms, st);
-  if (a.topk == 64 && Layout<D, 64, false>::fits(64)) return launch_tc_k<D, 64, false>(a, ctl, num_sms, st);
-  if (two_level && Layout<D, 128, false>::fits(a.topk)) return launch_tc_k<D, 128, false>(a, ctl, num_sms, st);
-  return launch_tc_k<D, 0, false>(a, ctl, num_sms, st);
+  switch (pick<D>(a.topk)) {
+    case TcKind::Split64: return launch_tc_k<D, 64, true>(a, ctl, num_sms, st);
+    case TcKind::Split128: return launch_tc_k<D, 128, true>(a, ctl, num_sms, st);
+    case TcKind::Split0: return launch_tc_k<D, 0, true>(a, ctl, num_sms, st);
+    case TcKind::Single64: return launch_tc_k<D, 64, false>(a, ctl, num_sms, st);
+    case TcKind::Single128: return launch_tc_k<D, 128, false>(a, ctl, num_sms, st);
+    default: return launch_tc_k<D, 0, false>(a, ctl, num_sms, st);
+  }
 }
 
 }  // namespace
@@ -514,6 +630,15 @@ bool attn_tc_supports(const AttnArgs& a) {
   if (a.d == 64) return Layout<64, 0, false>::fits(a.topk);
   if (a.d == 128) return Layout<128, 0, false>::fits(a.topk);
   return false;
+}
+
+size_t attn_tc_workspace_bytes(const AttnArgs& a, int num_sms) {
+  if (!attn_tc_supports(a)) return 0;
+  const bool split = a.d == 64 ? is_split(pick<64>(a.topk)) : is_split(pick<128>(a.topk));
+  if (!split) return 0;
+  const long long n_units = static_cast<long long>(a.B) * a.H * ((a.Lq + BM - 1) / BM);
+  const int grid = n_units < num_sms ? static_cast<int>(n_units) : num_sms;
+  return park_bytes(grid, a.topk);
 }
 
 int attn_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {

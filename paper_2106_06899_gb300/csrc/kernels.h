@@ -25,6 +25,9 @@ struct AttnArgs {
   int B, H, Lq, Lk, d, topk, chunk, causal, dtype;
   int32_t* idx;
   float* score;
+  // device scratch of the tcgen05 split kernel (attn_tc_workspace_bytes)
+  void* workspace = nullptr;
+  size_t workspace_bytes = 0;
 };
 
 struct FfnArgs {
@@ -47,6 +50,10 @@ struct FfnArgs {
 int attn_simt(const AttnArgs& a, cudaStream_t st);
 int attn_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st);
 bool attn_tc_supports(const AttnArgs& a);
+// Bytes of device scratch attn_tc needs for these arguments on a device with
+// num_sms SMs: the split kernel parks each unit's kept keys for its
+// epilogue warps (a fixed amount per CTA, nothing per query row); 0 otherwise.
+size_t attn_tc_workspace_bytes(const AttnArgs& a, int num_sms);
 
 size_t ffn_workspace_bytes(int N, int d_model, int d_ff, int topk);
 int ffn_tc(const FfnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st);

@@ -63,5 +63,16 @@ def test_ffn_argument_errors(lib):
     assert f(16, 16, 16, 16, 4, 64, 4096, 2000, None) == -2
 
 
-def test_attention_needs_no_workspace(lib):
-    assert T.topk_attn_workspace_bytes(1, 12, 65536, 65536, 64, 64, 1024, 1) == 0
+def test_attention_workspace_does_not_grow_with_the_sequence():
+    # the tcgen05 split kernel parks each work unit's kept keys for its epilogue warps: per CTA (at most
+    # one per SM) 4 heap warps x 2 slots x k keys x 32 rows x 8 bytes, plus a count per row; nothing per
+    # query row or key, so the scratch is the same at 8K, 64K and 1M tokens
+    sizes = {T.topk_attn_workspace_bytes(1, 12, L, L, 64, 64, 1024, 1) for L in (8192, 65536, 1 << 20)}
+    assert len(sizes) == 1
+    (ws,) = sizes
+    assert 0 < ws <= 1024 * (4 * 2 * 64 * 32 * 8 + 4 * 2 * 32 * 4)
+    # fp32 inputs and k above the tensor path's limit run the SIMT kernel, which needs none
+    assert T.topk_attn_workspace_bytes(1, 12, 65536, 65536, 64, 64, 1024, 0) == 0
+    assert T.topk_attn_workspace_bytes(1, 12, 4096, 4096, 64, 256, 1024, 1) == 0
+    # invalid arguments report 0
+    assert T.topk_attn_workspace_bytes(1, 12, 4096, 4096, 64, 0, 1024, 1) == 0

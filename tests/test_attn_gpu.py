@@ -161,8 +161,9 @@ def test_e2e_host_entry_in_head_slices_matches_device_entry(B, H, L, causal):
 
 
 def test_memory_is_linear_in_keys():
-    # Sec. 2.2: memory O(C L_K) for a fixed chunk; here the kernel holds no per-call device scratch at
-    # all, so the peak is the inputs and outputs themselves, linear in L_K
+    # Sec. 2.2: memory O(C L_K) for a fixed chunk; here the only device scratch is a fixed amount per
+    # CTA (the parked kept keys), the same for every L_K, so the peak is the inputs and outputs plus a
+    # constant: linear in L_K
     peaks = []
     for Lk in (8192, 16384, 32768, 65536):
         q, k, v = W.attention_inputs(1, 4, 1024, Lk, 64, dtype="bf16", seed=Lk)
@@ -177,7 +178,8 @@ def test_memory_is_linear_in_keys():
         T.topk_check()
         peaks.append(torch.cuda.max_memory_allocated() - base)
         assert torch.cuda.mem_get_info()[0] >= free0 - (dq.numel() * 2 * 4 + (64 << 20))
-        assert T.topk_attn_workspace_bytes(1, 4, 1024, Lk, 64, 64, 1024, 1) == 0
+        assert T.topk_attn_workspace_bytes(1, 4, 1024, Lk, 64, 64, 1024, 1) == T.topk_attn_workspace_bytes(
+            1, 4, 1024, 8192, 64, 64, 1024, 1)
         del dq, dk, dv, out
     d = np.diff(peaks)
     assert np.allclose(d[1:] / d[:-1], 2.0, rtol=0.02), peaks
