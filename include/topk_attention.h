@@ -165,13 +165,16 @@ size_t topk_ffn_workspace_bytes(int N, int d_model, int d_ff, int topk);
  * returning.  Sizes and dtypes as above.
  *   - topk_attn_fwd_host splits the B*H heads into up to 8 consecutive
  *     slices when there are enough query tiles (about 6 per SM per slice)
- *     and launches one call per slice on `stream`; each slice's inputs are
- *     copied on a copy stream of the library and its output copied back on
- *     another, so the copies of neighbouring slices overlap the kernels.
- *     The result is identical to one call over all heads.
+ *     and launches one call per slice, alternating between two compute
+ *     streams of the library (ordered after `stream`); each slice's inputs
+ *     are copied on a copy stream of the library and its output copied back
+ *     on another.  The copies of neighbouring slices overlap the kernels,
+ *     and a slice's kernel starts on the SMs the previous slice's last wave
+ *     leaves idle.  The result is identical to one call over all heads.
  *   - topk_ffn_fwd_host copies x and W1 first and W2 on a copy stream while
  *     the score and selection kernels run; the W2 gather waits for it.
- *   The copy streams are shared by all host-buffer calls on a device.
+ *   The library's streams are shared by all host-buffer calls on a device;
+ *   `stream` is synchronised, after it has waited for all of them.
  */
 int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq,
                        int Lk, int d, int topk, int chunk, int causal, int dtype, void* stream);

@@ -60,16 +60,19 @@ DevCtl make_ctl(DeviceState* s) {
   return c;
 }
 
-// Device memory the library allocates itself (feed-forward scratch, the
-// staging buffers of the host-buffer calls) comes from one stream-ordered
-// pool per device that keeps freed memory reserved for the next call, so a
-// steady stream of calls of one shape maps device memory once instead of on
-// every call.  Two non-blocking streams per device carry the host-buffer
-// calls' copies, so that they overlap the kernels on the caller's stream.
+// Device memory the library allocates itself (scratch, the staging buffers
+// of the host-buffer calls) comes from one stream-ordered pool per device
+// that keeps freed memory reserved for the next call, so a steady stream of
+// calls of one shape maps device memory once instead of on every call.  Two
+// non-blocking streams per device carry the host-buffer calls' copies, so
+// that they overlap the kernels, and two more take the attention call's head
+// slices in turn, so that the next slice's CTAs take the SMs that the
+// previous slice's last, partial wave leaves idle.
 struct HostPipe {
   std::once_flag once;
   cudaMemPool_t pool = nullptr;
   cudaStream_t h2d = nullptr, d2h = nullptr;
+  cudaStream_t comp[2] = {nullptr, nullptr};  // head slices alternate between these
   bool ok = false;
 };
 HostPipe g_pipe[kMaxDevices];
@@ -90,6 +93,8 @@ HostPipe* host_pipe() {
     if (cudaMemPoolSetAttribute(s.pool, cudaMemPoolAttrReleaseThreshold, &keep) != cudaSuccess) return;
     if (cudaStreamCreateWithFlags(&s.h2d, cudaStreamNonBlocking) != cudaSuccess) return;
     if (cudaStreamCreateWithFlags(&s.d2h, cudaStreamNonBlocking) != cudaSuccess) return;
+    for (cudaStream_t& c : s.comp)
+      if (cudaStreamCreateWithFlags(&c, cudaStreamNonBlocking) != cudaSuccess) return;
     s.ok = true;
   });
   return s.ok ? &s : nullptr;
@@ -295,19 +300,22 @@ int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, i
   P = P < 1 ? 1 : (P > BH ? BH : (P > kHostSlicesMax ? kHostSlicesMax : P));
 
   void *dq = nullptr, *dk = nullptr, *dv = nullptr, *dout = nullptr;
-  cudaEvent_t ready = nullptr, h2d_done = nullptr, d2h_done = nullptr;
+  cudaEvent_t ready = nullptr, h2d_done = nullptr, d2h_done = nullptr, comp_done[2] = {nullptr, nullptr};
   cudaEvent_t ev_in[kHostSlicesMax] = {}, ev_out[kHostSlicesMax] = {};
   auto mk = [](cudaEvent_t* e) { return cudaEventCreateWithFlags(e, cudaEventDisableTiming) == cudaSuccess; };
   bool good = pool_alloc(&dq, BH * qh, st) && pool_alloc(&dk, BH * kh, st) && pool_alloc(&dv, BH * kh, st) &&
-              pool_alloc(&dout, BH * qh, st) && mk(&ready) && mk(&h2d_done) && mk(&d2h_done);
+              pool_alloc(&dout, BH * qh, st) && mk(&ready) && mk(&h2d_done) && mk(&d2h_done) &&
+              mk(&comp_done[0]) && mk(&comp_done[1]);
   for (int s = 0; good && s < P; ++s) good = mk(&ev_in[s]) && mk(&ev_out[s]);
-  // the copy streams start once the allocations on `st` are in place
-  good = good && cudaEventRecord(ready, st) == cudaSuccess && cudaStreamWaitEvent(hp->h2d, ready, 0) == cudaSuccess &&
-         cudaStreamWaitEvent(hp->d2h, ready, 0) == cudaSuccess;
+  // the library streams start once the allocations on `st` are in place
+  good = good && cudaEventRecord(ready, st) == cudaSuccess;
+  for (cudaStream_t w : {hp->h2d, hp->d2h, hp->comp[0], hp->comp[1]})
+    good = good && cudaStreamWaitEvent(w, ready, 0) == cudaSuccess;
   if (!good) rc = TOPK_ERR_CUDA;
-  // slice s: its inputs on the h2d stream, its launch on `st` after them,
-  // its output on the d2h stream after the launch; the copies of slices
-  // s + 1 and s - 1 overlap the kernel of slice s
+  // slice s: its inputs on the h2d stream, its launch on compute stream
+  // s % 2 after them, its output on the d2h stream after the launch; the
+  // copies of slices s + 1 and s - 1 overlap the kernel of slice s, and the
+  // kernel of slice s + 1 starts on the SMs that slice s frees
   int launches = 0;
   for (int s = 0; rc == TOPK_OK && s < P; ++s) {
     const size_t h0 = static_cast<size_t>(static_cast<long long>(BH) * s / P);
@@ -323,27 +331,36 @@ int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, i
             cudaSuccess ||
         cudaMemcpyAsync(sv, static_cast<const uint8_t*>(v) + h0 * kh, nh * kh, cudaMemcpyHostToDevice, hp->h2d) !=
             cudaSuccess ||
-        cudaEventRecord(ev_in[s], hp->h2d) != cudaSuccess || cudaStreamWaitEvent(st, ev_in[s], 0) != cudaSuccess) {
+        cudaEventRecord(ev_in[s], hp->h2d) != cudaSuccess) {
       rc = TOPK_ERR_CUDA;
       break;
     }
-    rc = topk_attn_fwd(sq, sk, sv, so, 1, static_cast<int>(nh), Lq, Lk, d, topk, chunk, causal, dtype, stream);
+    cudaStream_t cs = hp->comp[s & 1];
+    if (cudaStreamWaitEvent(cs, ev_in[s], 0) != cudaSuccess) {
+      rc = TOPK_ERR_CUDA;
+      break;
+    }
+    rc = topk_attn_fwd(sq, sk, sv, so, 1, static_cast<int>(nh), Lq, Lk, d, topk, chunk, causal, dtype, cs);
     if (rc != TOPK_OK) break;
     launches += t_last_launches;
-    if (cudaEventRecord(ev_out[s], st) != cudaSuccess || cudaStreamWaitEvent(hp->d2h, ev_out[s], 0) != cudaSuccess ||
+    if (cudaEventRecord(ev_out[s], cs) != cudaSuccess || cudaStreamWaitEvent(hp->d2h, ev_out[s], 0) != cudaSuccess ||
         cudaMemcpyAsync(static_cast<uint8_t*>(out) + h0 * qh, so, nh * qh, cudaMemcpyDeviceToHost, hp->d2h) !=
             cudaSuccess) {
       rc = TOPK_ERR_CUDA;
       break;
     }
   }
-  // the buffers go back to the pool on `st` only after both copy streams
-  // are done with everything enqueued above
-  if (!(h2d_done && d2h_done && cudaEventRecord(h2d_done, hp->h2d) == cudaSuccess &&
-        cudaEventRecord(d2h_done, hp->d2h) == cudaSuccess && cudaStreamWaitEvent(st, h2d_done, 0) == cudaSuccess &&
-        cudaStreamWaitEvent(st, d2h_done, 0) == cudaSuccess)) {
-    cudaStreamSynchronize(hp->h2d);
-    cudaStreamSynchronize(hp->d2h);
+  // the buffers go back to the pool on `st` only after the copy and
+  // compute streams are done with everything enqueued above
+  bool joined = h2d_done && d2h_done && comp_done[0] && comp_done[1] &&
+                cudaEventRecord(h2d_done, hp->h2d) == cudaSuccess &&
+                cudaEventRecord(d2h_done, hp->d2h) == cudaSuccess &&
+                cudaEventRecord(comp_done[0], hp->comp[0]) == cudaSuccess &&
+                cudaEventRecord(comp_done[1], hp->comp[1]) == cudaSuccess;
+  for (cudaEvent_t e : {h2d_done, d2h_done, comp_done[0], comp_done[1]})
+    joined = joined && cudaStreamWaitEvent(st, e, 0) == cudaSuccess;
+  if (!joined) {
+    for (cudaStream_t w : {hp->h2d, hp->d2h, hp->comp[0], hp->comp[1]}) cudaStreamSynchronize(w);
     if (rc == TOPK_OK) rc = TOPK_ERR_CUDA;
   }
   if (dq) cudaFreeAsync(dq, st);
@@ -351,7 +368,7 @@ int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, i
   if (dv) cudaFreeAsync(dv, st);
   if (dout) cudaFreeAsync(dout, st);
   if (cudaStreamSynchronize(st) != cudaSuccess && rc == TOPK_OK) rc = TOPK_ERR_CUDA;
-  for (cudaEvent_t e : {ready, h2d_done, d2h_done})
+  for (cudaEvent_t e : {ready, h2d_done, d2h_done, comp_done[0], comp_done[1]})
     if (e) cudaEventDestroy(e);
   for (int s = 0; s < P; ++s) {
     if (ev_in[s]) cudaEventDestroy(ev_in[s]);
