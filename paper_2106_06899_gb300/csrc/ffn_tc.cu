@@ -54,7 +54,7 @@ constexpr int kFinalVec = 4;         // 16-byte candidate vectors each finalize 
 
 struct Plan {
   int n_rt, tiles, n_sl, n_units, cap;
-  size_t off_cnt, off_tau, off_kept, bytes;
+  size_t off_cnt, off_tau, off_part, off_kept, bytes;
 };
 
 Plan make_plan(int N, int d_model, int d_ff, int topk, int num_sms) {
@@ -89,7 +89,8 @@ Plan make_plan(int N, int d_model, int d_ff, int topk, int num_sms) {
   const size_t rows_sl = static_cast<size_t>(N) * p.n_sl;
   p.off_cnt = rows_sl * p.cap * sizeof(uint2);
   p.off_tau = p.off_cnt + rows_sl * sizeof(int);
-  p.off_kept = (p.off_tau + static_cast<size_t>(N) * sizeof(uint32_t) + 15) & ~size_t(15);
+  p.off_part = p.off_tau + static_cast<size_t>(N) * sizeof(uint32_t);
+  p.off_kept = (p.off_part + rows_sl * sizeof(uint32_t) + 15) & ~size_t(15);
   p.bytes = p.off_kept + static_cast<size_t>(N) * topk * sizeof(uint64_t);  // kept keys per token
   return p;
 }
@@ -127,6 +128,8 @@ struct RowCand {
   float base, width, inv_width;
   float L;            // valid lower bound of the row's k-th largest score
   float mn, mx;       // spread of the first k candidates
+  int kp;             // ceil(k / slices)
+  float Lp;           // valid lower bound of this slice's kp-th largest score
 
   __device__ __forceinline__ int bin(float s) const {
     const float f = fminf((s - base) * inv_width, static_cast<float>(NBINS - 1));
@@ -159,14 +162,16 @@ struct RowCand {
       return;
     }
     uint32_t acc = 0;
-    int bstar = 0;
+    int bstar = 0, bpart = -1;
     for (int b = NBINS - 1; b >= 0; --b) {
       acc += hist[b * BM];
+      if (bpart < 0 && acc >= static_cast<uint32_t>(kp)) bpart = b;  // kp <= k: found first
       if (acc >= static_cast<uint32_t>(k)) {
         bstar = b;
         break;
       }
     }
+    if (bpart >= 2) Lp = fmaxf(Lp, base + static_cast<float>(bpart - 1) * width);
     if (bstar >= 2) {
       L = fmaxf(L, base + static_cast<float>(bstar - 1) * width);
       if (bstar >= NBINS / 2) {  // slide the window up
@@ -241,7 +246,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     ffn_score_select_kernel(const __grid_constant__ CUtensorMap tmx, const __grid_constant__ CUtensorMap tmw,
                             int N, int d_model, int d_ff, int topk, int n_rt, int n_sl, int tiles, int n_units,
                             int cap, uint2* __restrict__ cand, int* __restrict__ cand_cnt,
-                            uint32_t* __restrict__ row_tau, DevCtl ctl) {
+                            uint32_t* __restrict__ row_tau, uint32_t* __restrict__ row_part, DevCtl ctl) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint32_t* hist_mem = reinterpret_cast<uint32_t*>(smem + OFF_HIST);
@@ -397,7 +402,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       rc.L = -INFINITY;
       rc.mn = INFINITY;
       rc.mx = -INFINITY;
-      uint32_t published = 0;
+      rc.kp = (topk + n_sl - 1) / n_sl;
+      rc.Lp = -INFINITY;
+      uint32_t published = 0, published_part = 0;
       for (int b = 0; b < NBINS; ++b) rc.hist[b * BM] = 0u;
 
       for (int kt = t0; kt < t1; ++kt, ++acc_it) {
@@ -439,6 +446,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lkey > published) {
           atomicMax(row_tau + grow, lkey);
           published = lkey;
+        }
+        // Pooled bound: every slice s of the row holds at least kp = ceil(k /
+        // slices) scores >= its Lp_s, so the row holds at least k scores >=
+        // min_s Lp_s, a valid bound of the row's k-th score however few of
+        // the row's top k each slice holds.  A slice publishes its Lp when it
+        // rises and raises the row's bound to the minimum of what every
+        // slice has published (0 = nothing yet; words only grow, so a stale
+        // one only makes the minimum smaller).
+        const uint32_t pkey = rc.Lp > -INFINITY ? ord_f32(rc.Lp) : 0u;
+        if (n_sl > 1 && pkey > published_part) {
+          const size_t r0 = static_cast<size_t>(grow) * n_sl;
+          atomicMax(row_part + r0 + sl, pkey);
+          published_part = pkey;
+          uint32_t mn = pkey;
+          for (int q = 0; q < n_sl && mn != 0u; ++q)
+            if (q != sl) mn = min(mn, *reinterpret_cast<volatile uint32_t*>(row_part + r0 + q));
+          if (mn != 0u) atomicMax(row_tau + grow, mn);
         }
         // ---- make room for the next tile: drop candidates below the bound (rare)
         if (kt + 1 < t1 && rc.cnt > rc.cap - NT) {
@@ -809,10 +833,12 @@ int ffn_tc(const FfnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
   uint2* cand = reinterpret_cast<uint2*>(ws);
   int* cnt = reinterpret_cast<int*>(ws + p.off_cnt);
   uint32_t* tau = reinterpret_cast<uint32_t*>(ws + p.off_tau);
+  uint32_t* part = reinterpret_cast<uint32_t*>(ws + p.off_part);
   CUtensorMap tmx, tmw;
   if (!make_tmap_bf16_2d(&tmx, a.x, a.d_model, a.N, BM)) return -1;
   if (!make_tmap_bf16_2d(&tmw, a.W1, a.d_model, a.d_ff, NT)) return -1;
   if (cudaMemsetAsync(tau, 0, static_cast<size_t>(a.N) * sizeof(uint32_t), st) != cudaSuccess) return -1;
+  if (cudaMemsetAsync(part, 0, static_cast<size_t>(a.N) * p.n_sl * sizeof(uint32_t), st) != cudaSuccess) return -1;
   // counts start at -1 ("not written"): the finalize reads no list whose count the first kernel did not set
   if (cudaMemsetAsync(cnt, 0xFF, static_cast<size_t>(a.N) * p.n_sl * sizeof(int), st) != cudaSuccess) return -1;
   if (cudaFuncSetAttribute(ffn_score_select_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -820,7 +846,7 @@ int ffn_tc(const FfnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
     return -1;
   const int grid = p.n_units < num_sms ? p.n_units : num_sms;
   ffn_score_select_kernel<<<grid, kThreads, SMEM_A, st>>>(tmx, tmw, a.N, a.d_model, a.d_ff, a.topk, p.n_rt, p.n_sl,
-                                                           p.tiles, p.n_units, p.cap, cand, cnt, tau, ctl);
+                                                           p.tiles, p.n_units, p.cap, cand, cnt, tau, part, ctl);
   if (cudaGetLastError() != cudaSuccess) return -1;
   constexpr size_t kFinalSmem = kFinalMaxCand * sizeof(uint64_t);
   if (cudaFuncSetAttribute(ffn_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,

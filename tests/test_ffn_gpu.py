@@ -66,12 +66,13 @@ def test_ffn_key_permutation_equivariance():
 
 
 def test_ffn_workspace_has_no_tokens_times_keys_term():
-    # scratch is N x slices x list capacity (slices <= 64, capacity <= 6k + 1024 whatever d_ff is), plus
-    # the k kept keys of each token (8 bytes each) for the gather
+    # scratch is N x slices x list capacity (slices <= 64, capacity <= 6k + 1024 whatever d_ff is), a count
+    # and a pooled-bound word per (token, slice), one bound word per token, plus the k kept keys of each
+    # token (8 bytes each) for the gather
     for N in (128, 1000, 4096):
         for dff in (4096, 65536, 1 << 20):
             ws = T.topk_ffn_workspace_bytes(N, 1024, dff, 512)
-            assert 0 < ws <= N * (64 * (6 * 512 + 1024) * 8 + 64 * 4 + 4 + 512 * 8) + 16
+            assert 0 < ws <= N * (64 * (6 * 512 + 1024) * 8 + 64 * 4 + 64 * 4 + 4 + 512 * 8) + 16
     assert T.topk_ffn_workspace_bytes(4096, 1024, 1 << 20, 512) < 4096 * (1 << 20)
 
 
