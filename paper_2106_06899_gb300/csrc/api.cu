@@ -242,13 +242,10 @@ size_t topk_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, int topk, 
   AttnArgs a{reinterpret_cast<void*>(16), reinterpret_cast<void*>(16), reinterpret_cast<void*>(16),
              reinterpret_cast<void*>(16), B, H, Lq, Lk, d, topk, chunk, 0, dtype, nullptr, nullptr};
   if (validate_attn(a) != TOPK_OK) return 0;
-  // sized for the current device; for a GB300 (152 SMs) when none is visible
-  int num_sms = kAssumedSms;
-  int dev = 0;
-  cudaDeviceProp p;
-  if (cudaGetDevice(&dev) == cudaSuccess && cudaGetDeviceProperties(&p, dev) == cudaSuccess)
-    num_sms = p.multiProcessorCount;
-  return attn_tc_workspace_bytes(a, num_sms);
+  // sized for the current device (the SM count the launch uses); for a
+  // GB300 (152 SMs) when none is visible
+  const DeviceState* dev = device_state();
+  return attn_tc_workspace_bytes(a, dev ? dev->num_sms : kAssumedSms);
 }
 
 size_t topk_ffn_workspace_bytes(int N, int d_model, int d_ff, int topk) {
