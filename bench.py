@@ -191,29 +191,65 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------ oracle timing
-def oracle_rate(w, seconds: float, seed_rows: int = 0):
-    """Oracle tokens/s on a bounded sample of rows of the workload (same inputs, all host cores)."""
+def oracle_rate(w, seconds: float, inputs, seed_rows: int = 0):
+    """Oracle tokens/s on a bounded sample of rows of the workload (same inputs, all host cores).
+
+    Returns (the cpu_baseline entry, the sampled rows, the oracle's result on them)."""
     import oracle
     from paper_2106_06899_gb300 import workloads as W
 
-    inputs = W.make_inputs(w)
     cores = oracle.hardware_threads()
 
     def run(nrows):
         rows = W.sample_rows(w.rows, nrows, seed=seed_rows).numpy()
         t0 = time.perf_counter()
         if w.kind == "ffn":
-            oracle.ffn(*inputs, w.topk, rows=rows)
+            res = oracle.ffn(*inputs, w.topk, rows=rows)
         else:
-            oracle.topk_attention(*inputs, w.topk, causal=w.causal, rows=rows)
-        return len(rows), time.perf_counter() - t0
+            res = oracle.topk_attention(*inputs, w.topk, causal=w.causal, rows=rows)
+        return rows, res, time.perf_counter() - t0
 
-    n, t = run(max(cores, 16))
-    target = max(int(n * seconds / max(t, 1e-3)), cores)
-    n, t = run(min(target, w.rows))
+    rows, res, t = run(max(cores, 16))
+    target = max(int(len(rows) * seconds / max(t, 1e-3)), cores)
+    rows, res, t = run(min(target, w.rows))
+    n = len(rows)
     per_token = w.H if w.kind == "attn" else 1
-    return {"value": (n / per_token) / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-            "sample": f"{n} of {w.rows} query rows (seeded sample), fp64 oracle, {t:.1f} s"}
+    entry = {"value": (n / per_token) / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+             "sample": f"{n} of {w.rows} query rows (seeded sample), fp64 oracle, {t:.1f} s"}
+    return entry, rows, res
+
+
+def parity_check(w, host, dev, out, rows, ref):
+    """The timed call's output on the oracle's sampled rows, under the parity rules of the tests
+    (oracle/parity.py): exact index sets outside near ties, every kept key valid, outputs within
+    tolerance.  The kept indices come from one extra call with index output, after the timed region
+    (selection is deterministic)."""
+    import torch
+
+    import oracle
+    from oracle.parity import check_rows
+    from paper_2106_06899_gb300 import topk as T
+
+    if w.kind == "ffn":
+        _, idx, score = T.ffn(dev[0], dev[1], dev[2], w.topk, return_indices=True)
+        q, k, v = (t[None, None] for t in host)
+        act, dtype, d = oracle.RELU, "bf16", w.d_model
+    else:
+        _, idx, score = T.attention(dev[0], dev[1], dev[2], w.topk, w.chunk, w.causal, return_indices=True)
+        q, k, v = host
+        act, dtype, d = oracle.SOFTMAX, w.dtype, w.d
+    T.topk_check()
+    r = torch.as_tensor(rows, dtype=torch.long, device=out.device)
+    gout = out.reshape(-1, d)[r].float().cpu().numpy()
+    gidx = idx.reshape(-1, w.topk)[r].cpu().numpy()
+    gscore = score.reshape(-1, w.topk)[r].cpu().numpy()
+    del idx, score
+    try:
+        st = check_rows(q=q, k=k, v=v, rows=rows, gpu_out=gout, gpu_idx=gidx, gpu_score=gscore, topk=w.topk,
+                        dtype=dtype, act=act, causal=w.causal, ref=ref)
+        return {"ok": True, **st}
+    except AssertionError as e:
+        return {"ok": False, "rows": len(rows), "error": str(e)}
 
 
 # ------------------------------------------------------------------ reference arm
@@ -395,12 +431,17 @@ def run_ours(args):
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clocks,
     }
+    parity_ok = True
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = oracle_rate(w, args.cpu_seconds)
+        line["cpu_baseline"], rows, ref = oracle_rate(w, args.cpu_seconds, host)
+        line["parity"] = parity_check(w, host, dev, out, rows, ref)
+        parity_ok = line["parity"]["ok"]
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
+    if not parity_ok:
+        sys.exit("parity check of the timed output failed: " + line["parity"]["error"])
 
 
 def main():

@@ -39,9 +39,10 @@
  *     *_workspace_bytes queries and is never proportional to Lq * Lk: a
  *     fixed amount per SM for attention, linear in the tokens for the
  *     feed-forward layer.  The pool keeps returned memory
- *     reserved for later calls (up to the largest amount in use at once)
- *     until the process exits, so that repeated calls do not map device
- *     memory again each time.
+ *     reserved for later calls (up to the largest amount in use at once),
+ *     so that repeated calls do not map device memory again each time, until
+ *     topk_pool_trim() hands it back or the process exits;
+ *     topk_pool_usage() reports it.
  *
  * Return codes: 0 on success, else one of the negative TOPK_ERR_* values;
  * topk_error_string() describes them.
@@ -67,9 +68,10 @@ enum {
   TOPK_ERR_CUDA = -3,        /* a CUDA runtime/driver call or a launch failed */
   TOPK_ERR_TIMEOUT = -4,     /* a device pipeline wait ran out its time limit; the
                                 kernel stopped early and its outputs are invalid */
-  TOPK_ERR_WORKSPACE = -5,   /* a per-row candidate list ran out of room (needs
-                                more keys tied within one bf16 step of the k-th
-                                score than the list holds); outputs invalid */
+  TOPK_ERR_WORKSPACE = -5,   /* an internal consistency check of the selection
+                                failed (no input is known to cause it; candidate
+                                lists are compacted exactly rather than overflow);
+                                outputs invalid */
   TOPK_ERR_NO_DEVICE = -6,   /* no usable sm_103 device */
   TOPK_ERR_SCRATCH_LIMIT = -7 /* the problem needs more scratch than the fixed buffer of
                                  topk_ffn_fwd_noalloc holds */
@@ -87,8 +89,9 @@ enum {
  *   Scratch: topk_attn_workspace_bytes() (a fixed amount per SM, or none).
  * Errors: TOPK_ERR_INVALID_ARG / TOPK_ERR_UNSUPPORTED before any launch;
  *         TOPK_ERR_CUDA if a launch fails (or the scratch cannot be had).
- *         Device-side timeouts surface on the next call or through
- *         topk_check().
+ *         A device-side timeout is not returned by this call (it returns
+ *         once the work is enqueued): topk_check() and the *_host calls
+ *         report it, from the device's error word (see topk_check).
  */
 int topk_attn_fwd(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk,
                   int d, int topk, int chunk, int causal, int dtype, void* stream);
@@ -181,9 +184,14 @@ int topk_attn_fwd_host(const void* q, const void* k, const void* v, void* out, i
 int topk_ffn_fwd_host(const void* x, const void* W1, const void* W2, void* out, int N, int d_model,
                       int d_ff, int topk, void* stream);
 
-/* Synchronises `stream` and returns the first device-side error recorded
- * since the last check (TOPK_ERR_TIMEOUT / TOPK_ERR_WORKSPACE), clearing it;
- * TOPK_ERR_CUDA if the stream itself reports an error; else TOPK_OK. */
+/* Synchronises `stream` and returns the device-side error recorded since the
+ * last check (TOPK_ERR_TIMEOUT before TOPK_ERR_WORKSPACE), clearing it;
+ * TOPK_ERR_CUDA if the stream itself reports an error; else TOPK_OK.
+ * The error word is ONE per device, shared by every stream and host thread
+ * that calls into the library on that device: an error raised by work on one
+ * stream is reported to (and cleared by) whichever caller checks first, and
+ * the *_host calls check it too.  Callers that share a device and need to
+ * tell their errors apart must serialise their calls and checks. */
 int topk_check(void* stream);
 
 /* Human-readable text for a return code (static storage). */
@@ -196,6 +204,19 @@ int topk_last_launch_count(void);
 /* Testing hook: sets the device-side wait limit in microseconds for later
  * calls (0 restores the default of 2 s) and returns the previous value. */
 long long topk_set_wait_limit_us(long long us);
+
+/* Device memory of the library's own stream-ordered pool on the current
+ * device (scratch of the device-pointer calls, staging buffers of the *_host
+ * calls): *used_high = the most bytes in use at once since the last reset,
+ * *reserved = bytes the pool holds now (in use or kept for later calls).
+ * Either pointer may be NULL; reset_high != 0 restarts the high-water mark
+ * after reading it.  Returns TOPK_ERR_NO_DEVICE without a usable device. */
+int topk_pool_usage(size_t* used_high, size_t* reserved, int reset_high);
+
+/* Hands the pool's reserved but unused memory back to the device.  Memory
+ * freed by enqueued work is released only once that work has completed:
+ * synchronise the streams that used the library first. */
+int topk_pool_trim(void);
 
 /* Testing hook: when `on` is non-zero, later tcgen05 attention launches
  * withhold their second key tile, so that the consumers' bounded waits run

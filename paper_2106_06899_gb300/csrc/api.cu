@@ -517,9 +517,31 @@ int topk_last_launch_count(void) { return t_last_launches; }
 
 long long topk_set_wait_limit_us(long long us) { return g_wait_limit_us.exchange(us < 0 ? 0 : us); }
 
-// Testing hook (not in the public header): makes the tcgen05 attention
-// producer withhold its second key tile so that the consumers' bounded waits
-// run out; returns the previous setting.
+// Testing hook: makes the tcgen05 attention producer withhold its second key
+// tile so that the consumers' bounded waits run out; returns the previous
+// setting.
 int topk_debug_skip_arrive(int on) { return g_debug_skip_arrive.exchange(on ? 1 : 0); }
+
+int topk_pool_usage(size_t* used_high, size_t* reserved, int reset_high) {
+  HostPipe* hp = host_pipe();
+  if (!hp) return TOPK_ERR_NO_DEVICE;
+  cuuint64_t hi = 0, res = 0;
+  if (cudaMemPoolGetAttribute(hp->pool, cudaMemPoolAttrUsedMemHigh, &hi) != cudaSuccess ||
+      cudaMemPoolGetAttribute(hp->pool, cudaMemPoolAttrReservedMemCurrent, &res) != cudaSuccess)
+    return TOPK_ERR_CUDA;
+  if (used_high) *used_high = static_cast<size_t>(hi);
+  if (reserved) *reserved = static_cast<size_t>(res);
+  if (reset_high) {
+    cuuint64_t zero = 0;  // the only value the high-water attributes accept
+    if (cudaMemPoolSetAttribute(hp->pool, cudaMemPoolAttrUsedMemHigh, &zero) != cudaSuccess) return TOPK_ERR_CUDA;
+  }
+  return TOPK_OK;
+}
+
+int topk_pool_trim(void) {
+  HostPipe* hp = host_pipe();
+  if (!hp) return TOPK_ERR_NO_DEVICE;
+  return cudaMemPoolTrimTo(hp->pool, 0) == cudaSuccess ? TOPK_OK : TOPK_ERR_CUDA;
+}
 
 }  // extern "C"

@@ -9,14 +9,23 @@
 //    128-token tile x one slice of the d_ff keys.  TMA streams x and W1
 //    chunks of 64 columns; tcgen05.mma accumulates the [128 x 256] score
 //    tile in TMEM (double buffered); thread t of the selection warps owns
-//    token row t.  Each row keeps a valid lower bound L of its k-th largest
-//    score and appends every score s >= L to its candidate list for this
-//    slice (device workspace, linear in tokens).  L comes from a 64-bin
+//    token row t.  Each row keeps a lower bound L of its slice's k-th
+//    largest score and appends a score s to its candidate list for this
+//    slice (device workspace, linear in tokens) only if s > L and s >= Lg,
+//    Lg being the row's bound shared across slices.  L comes from a 64-bin
 //    histogram of the candidates' scores kept in shared memory: the lower
 //    edge of the highest bin with k candidates at or above it is <= the
-//    k-th largest score, so raising L to it never drops a true top-k key.
-//    Rows also share L across slices through one word per row (the k-th
-//    largest of any subset of keys is <= that of all keys).
+//    k-th largest score.  Keys of a slice stream in ascending index order,
+//    so the k candidates behind L all have lower indices than any key still
+//    to come: a later key scoring exactly L ranks below all of them (ties go
+//    to the lower index) and is not appended.  A row of equal scores (an
+//    all-zero token, say) thus keeps about k candidates per slice, not all
+//    of its keys.  Rows share a bound across slices through one word per
+//    row (the k-th largest of any subset of keys is <= that of all keys);
+//    its supporting keys may sit in other slices, at higher indices, so it
+//    is applied non-strictly.  When bound filtering cannot free room in a
+//    list, the list is compacted exactly to its k best entries and L rises
+//    to the k-th of them (same argument), so no input overflows a list.
 // 2. ffn_finalize_kernel (one CTA per token).  Reads the row's candidates
 //    from every slice and keeps the exact top-k by the total order (score
 //    descending, index ascending), sorted, in the workspace.
@@ -120,13 +129,13 @@ __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, const
 // that fp32 rounding of the bin index can never place a candidate above
 // the bound it supports.
 struct RowCand {
-  uint2* list;        // this (row, slice)'s candidate list
+  uint2* list;        // this (row, slice)'s candidate list, ascending key index
   uint32_t* hist;     // &hist[bin 0][row], stride BM
   int cap, cnt, k;
-  bool dead;          // list overflowed (outputs invalid, error flagged)
   bool hist_on;
   float base, width, inv_width;
-  float L;            // valid lower bound of the row's k-th largest score
+  float L;            // this slice already holds k keys scoring >= L, all of lower index than
+                      // any key still to come: a later key must beat L strictly
   float mn, mx;       // spread of the first k candidates
   int kp;             // ceil(k / slices)
   float Lp;           // valid lower bound of this slice's kp-th largest score
@@ -188,10 +197,14 @@ struct RowCand {
   uint32_t* rj;
   int rc;
 
+  // A score qualifies for the list if it reaches the shared bound Lg and
+  // beats the slice's own bound Ls strictly (see L above).
+  __device__ __forceinline__ static bool keep(float s, float Lg, float Ls) { return s >= Lg && s > Ls; }
+
   // Expand every lane's records into its candidate list, lanes in lockstep:
-  // per record slot each lane forms the mask of its elements >= Lf, then the
-  // warp appends one element per lane per step.
-  __device__ __forceinline__ void flush(float Lf, bool active) {
+  // per record slot each lane forms the mask of its qualifying elements,
+  // then the warp appends one element per lane per step.
+  __device__ __forceinline__ void flush(float Lg, float Ls, bool active) {
     const int mxr = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(active ? rc : 0));
     for (int i = 0; i < mxr; ++i) {
       unsigned msk = 0;
@@ -200,8 +213,9 @@ struct RowCand {
         const float4 a = rlo[i * BM];
         const float4 b = rhi[i * BM];
         j0 = rj[i * BM];
-        msk = (a.x >= Lf ? 1u : 0u) | (a.y >= Lf ? 2u : 0u) | (a.z >= Lf ? 4u : 0u) | (a.w >= Lf ? 8u : 0u) |
-              (b.x >= Lf ? 16u : 0u) | (b.y >= Lf ? 32u : 0u) | (b.z >= Lf ? 64u : 0u) | (b.w >= Lf ? 128u : 0u);
+        msk = (keep(a.x, Lg, Ls) ? 1u : 0u) | (keep(a.y, Lg, Ls) ? 2u : 0u) | (keep(a.z, Lg, Ls) ? 4u : 0u) |
+              (keep(a.w, Lg, Ls) ? 8u : 0u) | (keep(b.x, Lg, Ls) ? 16u : 0u) | (keep(b.y, Lg, Ls) ? 32u : 0u) |
+              (keep(b.z, Lg, Ls) ? 64u : 0u) | (keep(b.w, Lg, Ls) ? 128u : 0u);
       }
       while (__any_sync(0xffffffffu, msk != 0)) {
         if (msk) {
@@ -216,10 +230,10 @@ struct RowCand {
     rc = 0;
   }
 
-  // Offer 64 scores (key indices j0..j0+63) against the bound Lf: each group
-  // of 8 whose maximum reaches Lf becomes one record (NaN, used for keys past
-  // d_ff, never does).
-  __device__ __forceinline__ void offer64(const float (&v)[64], uint32_t j0, float Lf, bool active) {
+  // Offer 64 scores (key indices j0..j0+63): each group of 8 whose maximum
+  // qualifies (keep()) becomes one record (NaN, used for keys past d_ff,
+  // never does).
+  __device__ __forceinline__ void offer64(const float (&v)[64], uint32_t j0, float Lg, float Ls, bool active) {
     float m[8];
 #pragma unroll
     for (int g = 0; g < 8; ++g)
@@ -229,7 +243,7 @@ struct RowCand {
       int r = rc;
 #pragma unroll
       for (int g = 0; g < 8; ++g) {
-        if (m[g] >= Lf) {
+        if (keep(m[g], Lg, Ls)) {
           rlo[r * BM] = make_float4(v[8 * g], v[8 * g + 1], v[8 * g + 2], v[8 * g + 3]);
           rhi[r * BM] = make_float4(v[8 * g + 4], v[8 * g + 5], v[8 * g + 6], v[8 * g + 7]);
           rj[r * BM] = j0 + 8 * g;
@@ -238,7 +252,52 @@ struct RowCand {
       }
       rc = r;
     }
-    if (__any_sync(0xffffffffu, active && rc > GR - 8)) flush(Lf, active);
+    if (__any_sync(0xffffffffu, active && rc > GR - 8)) flush(Lg, Ls, active);
+  }
+
+  // The list's exact top k by the total order (score descending, index
+  // ascending), in place, keeping list order; L rises to the k-th score.
+  // Called when filtering by the bound frees too little room (many keys
+  // scoring within a histogram bin of the k-th): every dropped entry ranks
+  // below k entries of the list, and so does any later key that does not
+  // beat L strictly (the k kept entries have lower indices).  Needs cnt > k.
+  // The k-th largest score is found bit by bit (MSB first) on the ordered
+  // score keys, below the prefix that every entry shares.
+  __device__ void compact_exact() {
+    uint32_t lo = 0xFFFFFFFFu, hi = 0u;
+    for (int i = 0; i < cnt; ++i) {
+      const uint32_t o = ord_f32(__uint_as_float(list[i].x));
+      lo = min(lo, o);
+      hi = max(hi, o);
+    }
+    uint32_t t = 0;
+    if (lo == hi) {
+      t = lo;
+    } else {
+      const int top = 31 - __clz(lo ^ hi);  // highest bit where entries differ
+      t = hi & ~((2u << top) - 1u);         // the shared prefix (bit `top` and below cleared)
+      for (int b = top; b >= 0; --b) {
+        const uint32_t cand = t | (1u << b);
+        int c = 0;
+        for (int i = 0; i < cnt; ++i) c += ord_f32(__uint_as_float(list[i].x)) >= cand ? 1 : 0;
+        if (c >= k) t = cand;
+      }
+    }
+    // t: ordered key of the k-th largest score.  Keep every entry above it and,
+    // in list (= index) order, as many entries equal to it as make k.
+    int above = 0;
+    for (int i = 0; i < cnt; ++i) above += ord_f32(__uint_as_float(list[i].x)) > t ? 1 : 0;
+    int eq_left = k - above;
+    int w = 0;
+    for (int i = 0; i < cnt; ++i) {
+      const uint2 e = list[i];
+      const uint32_t o = ord_f32(__uint_as_float(e.x));
+      const bool take = o > t || (o == t && eq_left > 0);
+      if (o == t && take) --eq_left;
+      if (take) list[w++] = e;
+    }
+    cnt = w;
+    L = fmaxf(L, unord_f32(t));
   }
 };
 
@@ -394,7 +453,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       const size_t rs = static_cast<size_t>(row_ok ? grow : 0) * n_sl + sl;
       rc.list = cand + rs * cap;
       rc.cnt = 0;
-      rc.dead = false;
       rc.hist_on = false;
       rc.base = 0.0f;
       rc.width = 1.0f;
@@ -411,7 +469,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         // the bound shared by the other slices of this row
         const uint32_t shared_key = row_ok ? *reinterpret_cast<volatile uint32_t*>(row_tau + grow) : 0u;
         const float Lg = shared_key ? unord_f32(shared_key) : -INFINITY;
-        const float L = fmaxf(rc.L, Lg);
+        const float Ls = rc.L;  // refresh() moves it only after this tile's flush
         const int b = acc_it & 1;
         if (!warp_wait(&acc_full[b], (acc_it >> 1) & 1u, ctl, abort_flag)) {
           ok = false;
@@ -436,11 +494,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             for (int e = 0; e < 64; ++e)
               if (j0 + e >= static_cast<uint32_t>(d_ff)) v[e] = __uint_as_float(0x7fc00000u);  // NaN: never kept
           }
-          rc.offer64(v, j0, L, row_ok && !rc.dead);
+          rc.offer64(v, j0, Lg, Ls, row_ok);
         }
         // the tile's pending groups go to the list before the bound moves
-        if (__any_sync(0xffffffffu, row_ok && !rc.dead && rc.rc > 0)) rc.flush(L, row_ok && !rc.dead);
-        if (!row_ok || rc.dead) continue;
+        if (__any_sync(0xffffffffu, row_ok && rc.rc > 0)) rc.flush(Lg, Ls, row_ok);
+        if (!row_ok) continue;
         rc.refresh();
         const uint32_t lkey = rc.L > -INFINITY ? ord_f32(rc.L) : 0u;
         if (lkey > published) {
@@ -464,7 +522,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (q != sl) mn = min(mn, *reinterpret_cast<volatile uint32_t*>(row_part + r0 + q));
           if (mn != 0u) atomicMax(row_tau + grow, mn);
         }
-        // ---- make room for the next tile: drop candidates below the bound (rare)
+        // ---- make room for the next tile (rare): drop candidates below the
+        // bound (entries equal to it may be the row's top k and stay); if that
+        // is not enough, keep exactly the list's k best.  cap >= k + 2 NT
+        // whenever a slice has more keys than cap (make_plan), so either way
+        // the next tile's NT keys fit.
         if (kt + 1 < t1 && rc.cnt > rc.cap - NT) {
           const float Lc = fmaxf(rc.L, Lg);
           int w = 0;
@@ -473,14 +535,11 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (__uint_as_float(e.x) >= Lc) rc.list[w++] = e;
           }
           rc.cnt = w;
-          if (w > rc.cap - NT) {
-            rc.dead = true;
-            atomicOr(ctl.error, kDevErrWorkspace);
-          }
+          if (w > rc.cap - NT) rc.compact_exact();
         }
       }
       if (!ok) break;
-      if (row_ok) cand_cnt[rs] = rc.dead ? -1 : min(rc.cnt, rc.cap);
+      if (row_ok) cand_cnt[rs] = rc.cnt;
     }
   }
 
@@ -498,10 +557,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 // MSB-first radix select over their ordered score keys (11, 11 and 10 bits;
 // histograms in shared memory, increments aggregated per warp with
 // __match_any_sync so that equal digits do not serialise) finds the exact
-// k-th largest score t and how many keys equal to t are needed.  The kept
-// set is every key with score > t plus the needed keys equal to t with the
-// lowest indices (the tie rule); it is then sorted best first with a
-// bitonic sort of the packed keys.
+// k-th largest score t and how many keys scoring t the kept set takes.  When
+// more keys score t than that, the tie rule (lower index first) decides:
+// a second radix select, over the complemented indices of the keys scoring
+// t, finds the index where the kept ties stop.  The kept set -- every key
+// above t plus the chosen ties -- is sorted best first with a bitonic sort
+// of the packed keys.  When everything at or above the k-th key's first
+// digit fits in shared memory, it is collected and sorted there directly.
 constexpr int kHistBins = 2048;
 
 __device__ __forceinline__ void warp_hist_add(uint32_t* hist, uint32_t d, bool valid) {
@@ -521,19 +583,42 @@ __device__ __forceinline__ int warp_append(int* counter, bool take) {
   return take ? base + __popc(bal & ((1u << lane) - 1u)) : -1;
 }
 
+// Bitonic sort of keys[0, n) in shared memory, descending; slots n .. next
+// power of two are padded with 0 (which ranks last).  All threads call it.
+__device__ __forceinline__ void bitonic_desc(uint64_t* keys, int n) {
+  int m = 1;
+  while (m < n) m <<= 1;
+  for (int i = n + static_cast<int>(threadIdx.x); i < m; i += blockDim.x) keys[i] = 0ull;
+  __syncthreads();
+  for (int size = 2; size <= m; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = threadIdx.x; i < (m >> 1); i += blockDim.x) {
+        const int lo = 2 * i - (i & (stride - 1));
+        const int hi = lo + stride;
+        const bool desc = (lo & size) == 0;
+        const uint64_t a = keys[lo], b = keys[hi];
+        if ((a < b) == desc) {
+          keys[lo] = b;
+          keys[hi] = a;
+        }
+      }
+      __syncthreads();
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kFinalThreads)
     ffn_finalize_kernel(uint64_t* __restrict__ kept, int topk, int n_sl, int cap, const uint2* __restrict__ cand,
                         const int* __restrict__ cand_cnt, const uint32_t* __restrict__ row_tau,
                         int32_t* __restrict__ idx, float* __restrict__ score, DevCtl ctl) {
   extern __shared__ uint64_t keys[];  // [kFinalMaxCand]; the first kHistBins words double as the histogram
   __shared__ uint32_t csum[kFinalThreads];
-  __shared__ int n_keys, n_ties, bad, sh_digit, sh_above;
+  __shared__ int n_keys, bad, sh_digit, sh_above, sh_count;
   uint32_t* hist = reinterpret_cast<uint32_t*>(keys);
   const int row = blockIdx.x;
   const int tid = threadIdx.x;
   if (tid == 0) {
     n_keys = 0;
-    n_ties = 0;
     bad = 0;
   }
   __syncthreads();
@@ -541,7 +626,7 @@ __global__ void __launch_bounds__(kFinalThreads)
   const float L = tk ? unord_f32(tk) : -INFINITY;
   for (int sl = tid; sl < n_sl; sl += kFinalThreads) {
     const int c = cand_cnt[static_cast<size_t>(row) * n_sl + sl];
-    if (c < 0 || c > cap) bad = 1;  // overflowed, or never written (first kernel stopped early)
+    if (c < 0 || c > cap) bad = 1;  // never written: the first kernel stopped early (a timeout)
   }
   __syncthreads();
   if (bad) {
@@ -578,21 +663,18 @@ __global__ void __launch_bounds__(kFinalThreads)
       }
     }
   };
-  // radix select: the k-th largest ordered key among the candidates >= L
-  uint32_t prefix = 0, pmask = 0;
-  int remaining = topk;
-  bool direct = false;
-  const int shifts[3] = {21, 10, 0};
-  const uint32_t dmasks[3] = {0x7FFu, 0x7FFu, 0x3FFu};
-#pragma unroll
-  for (int pass = 0; pass < 3; ++pass) {
+  // One MSB-first radix digit: over the candidates with mine(o, j) whose
+  // value val(o, j) matches `prefix` on `pmask`, histogram the digit
+  // (val >> sh) & dm and find the digit holding the remaining-th largest
+  // value.  Sets sh_digit (-1 if fewer than `remaining` such candidates),
+  // sh_above (candidates in higher digits) and sh_count (in that digit).
+  auto radix_digit = [&](auto&& mine, auto&& val, uint32_t prefix, uint32_t pmask, int sh, uint32_t dm,
+                         int remaining) {
     for (int i = tid; i < kHistBins; i += kFinalThreads) hist[i] = 0u;
     __syncthreads();
-    const int sh = shifts[pass];
-    const uint32_t dm = dmasks[pass];
-    for_each([&](bool valid, uint32_t o, uint32_t) {
-      const bool mine = valid && (o & pmask) == prefix;
-      warp_hist_add(hist, (o >> sh) & dm, mine);
+    for_each([&](bool valid, uint32_t o, uint32_t j) {
+      const uint32_t x = val(o, j);
+      warp_hist_add(hist, (x >> sh) & dm, valid && mine(o, j) && (x & pmask) == prefix);
     });
     __syncthreads();
     // chunk sums from the top bin down, then one thread locates the digit
@@ -623,17 +705,31 @@ __global__ void __launch_bounds__(kFinalThreads)
       }
       sh_digit = digit;
       sh_above = static_cast<int>(cum);
+      sh_count = digit >= 0 ? static_cast<int>(hist[digit]) : 0;
     }
     __syncthreads();
-    if (sh_digit < 0) {  // fewer candidates than k: cannot happen unless the lists are inconsistent
+  };
+  const int shifts[3] = {21, 10, 0};
+  const uint32_t dmasks[3] = {0x7FFu, 0x7FFu, 0x3FFu};
+  auto any = [](uint32_t, uint32_t) { return true; };
+  auto score_of = [](uint32_t o, uint32_t) { return o; };
+  // radix select: the k-th largest ordered score among the candidates
+  uint32_t prefix = 0, pmask = 0;
+  int remaining = topk, n_eq = 0;
+  bool direct = false;
+#pragma unroll 1
+  for (int pass = 0; pass < 3; ++pass) {
+    radix_digit(any, score_of, prefix, pmask, shifts[pass], dmasks[pass], remaining);
+    const int digit = sh_digit, above = sh_above, count = sh_count;
+    if (digit < 0) {  // fewer candidates than k: cannot happen unless the lists are inconsistent
       if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
       return;
     }
-    prefix |= static_cast<uint32_t>(sh_digit) << sh;
-    pmask |= dm << sh;
-    remaining -= sh_above;
-    const int kept_or_open = (topk - remaining) + static_cast<int>(hist[sh_digit]);
-    __syncthreads();
+    prefix |= static_cast<uint32_t>(digit) << shifts[pass];
+    pmask |= dmasks[pass] << shifts[pass];
+    remaining -= above;
+    n_eq = count;
+    const int kept_or_open = (topk - remaining) + count;
     if (pass == 0 && kept_or_open <= kFinalMaxCand) {
       // everything at or above the k-th key's leading 11 bits fits in shared
       // memory: collect it and finish there (one more read of the lists)
@@ -647,97 +743,47 @@ __global__ void __launch_bounds__(kFinalThreads)
         if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
         return;
       }
-      int m2 = 1;
-      while (m2 < nc) m2 <<= 1;
-      for (int i = nc + tid; i < m2; i += kFinalThreads) keys[i] = 0ull;
-      __syncthreads();
-      for (int size = 2; size <= m2; size <<= 1) {
-        for (int stride = size >> 1; stride > 0; stride >>= 1) {
-          for (int i = tid; i < (m2 >> 1); i += kFinalThreads) {
-            const int lo = 2 * i - (i & (stride - 1));
-            const int hi = lo + stride;
-            const bool desc = (lo & size) == 0;
-            const uint64_t a = keys[lo], b = keys[hi];
-            if ((a < b) == desc) {
-              keys[lo] = b;
-              keys[hi] = a;
-            }
-          }
-          __syncthreads();
-        }
-      }
+      bitonic_desc(keys, nc);
       direct = true;  // keys[0 .. topk) are the kept keys, best first
       break;
     }
   }
   if (!direct) {
-  // prefix = ordered key of the k-th largest score; `remaining` keys equal to it are kept
-  const uint32_t thr = prefix;
-  uint32_t* ties = reinterpret_cast<uint32_t*>(keys + topk);  // indices of keys equal to thr
-  const int tie_cap = (kFinalMaxCand - topk) * 2;
-  for_each([&](bool valid, uint32_t o, uint32_t j) {
-    const int pa = warp_append(&n_keys, valid && o > thr);
-    if (pa >= 0 && pa < topk) keys[pa] = (static_cast<uint64_t>(o) << 32) | static_cast<uint64_t>(~j);
-    const int pt = warp_append(&n_ties, valid && o == thr);
-    if (pt >= 0 && pt < tie_cap) ties[pt] = j;
-  });
-  __syncthreads();
-  const int na = n_keys, nt = n_ties;
-  if (na + remaining != topk || nt < remaining || nt > tie_cap) {
-    if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
-    return;
-  }
-  // the `remaining` lowest indices among the ties (ascending bitonic sort of the tie indices)
-  if (nt > remaining) {
-    int m = 1;
-    while (m < nt) m <<= 1;
-    if (m > tie_cap) {
+    // prefix: ordered key t of the k-th largest score; the kept set takes
+    // `remaining` of the n_eq keys scoring t, those of lowest index
+    const uint32_t thr = prefix;
+    uint32_t jsel = 0;  // a key scoring t is kept iff ~index >= jsel
+    if (n_eq > remaining) {
+      auto is_tie = [thr](uint32_t o, uint32_t) { return o == thr; };
+      auto inv_index = [](uint32_t, uint32_t j) { return ~j; };
+      uint32_t p2 = 0, m2 = 0;
+      int rem2 = remaining;
+#pragma unroll 1
+      for (int pass = 0; pass < 3; ++pass) {
+        radix_digit(is_tie, inv_index, p2, m2, shifts[pass], dmasks[pass], rem2);
+        if (sh_digit < 0) {
+          if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
+          return;
+        }
+        p2 |= static_cast<uint32_t>(sh_digit) << shifts[pass];
+        m2 |= dmasks[pass] << shifts[pass];
+        rem2 -= sh_above;
+      }
+      jsel = p2;  // the remaining-th largest ~index among the ties (indices are distinct)
+    }
+    __syncthreads();
+    if (tid == 0) n_keys = 0;
+    __syncthreads();
+    for_each([&](bool valid, uint32_t o, uint32_t j) {
+      const int pa = warp_append(&n_keys, valid && (o > thr || (o == thr && ~j >= jsel)));
+      if (pa >= 0 && pa < topk) keys[pa] = (static_cast<uint64_t>(o) << 32) | static_cast<uint64_t>(~j);
+    });
+    __syncthreads();
+    if (n_keys != topk) {
       if (tid == 0) atomicOr(ctl.error, kDevErrWorkspace);
       return;
     }
-    for (int i = nt + tid; i < m; i += kFinalThreads) ties[i] = 0xFFFFFFFFu;
-    __syncthreads();
-    for (int size = 2; size <= m; size <<= 1) {
-      for (int stride = size >> 1; stride > 0; stride >>= 1) {
-        for (int i = tid; i < (m >> 1); i += kFinalThreads) {
-          const int lo = 2 * i - (i & (stride - 1));
-          const int hi = lo + stride;
-          const bool asc = (lo & size) == 0;
-          const uint32_t x = ties[lo], y = ties[hi];
-          if ((x > y) == asc) {
-            ties[lo] = y;
-            ties[hi] = x;
-          }
-        }
-        __syncthreads();
-      }
-    }
-  }
-  __syncthreads();
-  for (int t = tid; t < remaining; t += kFinalThreads)
-    keys[na + t] = (static_cast<uint64_t>(thr) << 32) | static_cast<uint64_t>(~ties[t]);
-  __syncthreads();
-  const int n = topk;
-  // bitonic sort of the k kept keys, descending (padding keys rank last)
-  int m = 1;
-  while (m < n) m <<= 1;
-  for (int i = n + tid; i < m; i += kFinalThreads) keys[i] = 0ull;
-  __syncthreads();
-  for (int size = 2; size <= m; size <<= 1) {
-    for (int stride = size >> 1; stride > 0; stride >>= 1) {
-      for (int i = tid; i < (m >> 1); i += kFinalThreads) {
-        const int lo = 2 * i - (i & (stride - 1));
-        const int hi = lo + stride;
-        const bool desc = (lo & size) == 0;
-        const uint64_t a = keys[lo], b = keys[hi];
-        if ((a < b) == desc) {
-          keys[lo] = b;
-          keys[hi] = a;
-        }
-      }
-      __syncthreads();
-    }
-  }
+    bitonic_desc(keys, topk);
   }
   // the kept keys, in selection order, for the gather kernel
   for (int t = tid; t < topk; t += kFinalThreads) kept[static_cast<size_t>(row) * topk + t] = keys[t];

@@ -56,10 +56,12 @@ def lib() -> ctypes.CDLL:
             L.topk_set_wait_limit_us.argtypes = [ctypes.c_longlong]
             L.topk_set_wait_limit_us.restype = ctypes.c_longlong
             L.topk_debug_skip_arrive.argtypes = [i32]
+            L.topk_pool_usage.argtypes = [ctypes.POINTER(sz), ctypes.POINTER(sz), i32]
+            L.topk_pool_trim.argtypes = []
             for f in ("topk_attn_fwd", "topk_attn_fwd_indices", "topk_ffn_fwd", "topk_ffn_fwd_indices",
                       "topk_attn_fwd_host", "topk_ffn_fwd_host", "topk_ffn_fwd_noalloc", "topk_check",
                       "topk_last_launch_count",
-                      "topk_debug_skip_arrive"):
+                      "topk_debug_skip_arrive", "topk_pool_usage", "topk_pool_trim"):
                 getattr(L, f).restype = i32
             _lib = L
     return _lib
@@ -203,6 +205,19 @@ def topk_last_launch_count() -> int:
 
 def topk_set_wait_limit_us(us: int) -> int:
     return int(lib().topk_set_wait_limit_us(int(us)))
+
+
+def topk_pool_usage(reset_high: bool = False) -> tuple[int, int]:
+    """(bytes in use at most since the last reset, bytes reserved now) of the library's own
+    device-memory pool on the current device."""
+    hi, res = ctypes.c_size_t(0), ctypes.c_size_t(0)
+    _check(lib().topk_pool_usage(ctypes.byref(hi), ctypes.byref(res), int(bool(reset_high))), "topk_pool_usage")
+    return int(hi.value), int(res.value)
+
+
+def topk_pool_trim() -> None:
+    """Hand the pool's reserved but unused device memory back (synchronise the streams first)."""
+    _check(lib().topk_pool_trim(), "topk_pool_trim")
 
 
 # convenience wrappers that allocate the outputs ---------------------------------------------

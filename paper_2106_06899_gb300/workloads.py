@@ -116,13 +116,23 @@ def attention_inputs(B, H, Lq, Lk, d, *, dtype="bf16", seed=0, dist="normal"):
     return (q * scale).to(td).contiguous(), (k * scale).to(td).contiguous(), v.to(td).contiguous()
 
 
-def ffn_inputs(N, d_model, d_ff, *, dtype="bf16", seed=0):
-    """(x [N,d_model], W1 [d_ff,d_model], W2 [d_ff,d_model]) on the CPU in ``dtype``."""
+def ffn_inputs(N, d_model, d_ff, *, dtype="bf16", seed=0, dist="ffn"):
+    """(x [N,d_model], W1 [d_ff,d_model], W2 [d_ff,d_model]) on the CPU in ``dtype``.
+
+    ``dist="integer"`` draws x and W1 from the integers -2..2 instead (W2 stays
+    normal): every score is then an exact integer in any precision, so the
+    k-th score is shared by many keys and both sides see the same ties."""
     g = torch.Generator().manual_seed(int(seed))
     td = _torch_dtype(dtype)
-    x = torch.randn(N, d_model, generator=g)
     std = 1.0 / math.sqrt(d_model)
-    w1 = torch.randn(d_ff, d_model, generator=g) * std
+    if dist == "ffn":
+        x = torch.randn(N, d_model, generator=g)
+        w1 = torch.randn(d_ff, d_model, generator=g) * std
+    elif dist == "integer":
+        x = torch.randint(-2, 3, (N, d_model), generator=g).float()
+        w1 = torch.randint(-2, 3, (d_ff, d_model), generator=g).float()
+    else:
+        raise ValueError(f"unknown distribution {dist!r}")
     w2 = torch.randn(d_ff, d_model, generator=g) * std
     return x.to(td).contiguous(), w1.to(td).contiguous(), w2.to(td).contiguous()
 

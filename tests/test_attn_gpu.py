@@ -46,10 +46,18 @@ def test_tiny_fp32_all_rows():
     assert st["rows"] == 512
 
 
+# Exact-set floors for the full-size workloads.  Rows with a clear gap between the k-th and (k+1)-th
+# oracle scores must match exactly (check_rows asserts that); near-tie rows (bert_base ~11 %, long_65k
+# ~50 %, causal_16k ~47 % of rows, from the oracle) may differ only where fp32 rounding reorders scores
+# within about 1e-6 relative, which is rare.  The floors below are well under what that allows.
+EXACT_FLOOR = {"bert_base": 0.95, "long_65k": 0.95, "causal_16k": 0.95}
+
+
 def test_bert_base_all_rows():
     w, (q, k, v) = _workload("bert_base")
     st = _check(q, k, v, w.topk, "bf16", chunk=w.chunk)
-    assert st["exact_set_frac"] > 0.5
+    print(f"bert_base: {st}")
+    assert st["exact_set_frac"] >= EXACT_FLOOR["bert_base"]
 
 
 def test_bert_base_all_keys_is_plain_attention():
@@ -64,21 +72,33 @@ def test_bert_base_all_keys_is_plain_attention():
 
 
 def test_long_65k_sampled_rows():
+    # 4096 seeded rows of the 786,432, plus every row of one 128-query tile (the kernel's work unit)
     w, (q, k, v) = _workload("long_65k")
-    rows = W.sample_rows(w.rows, 96, seed=2).numpy()
+    tile = 5 * w.Lq + 128 * 300 + np.arange(128)  # head 5, query tile 300
+    rows = np.unique(np.concatenate([W.sample_rows(w.rows, 4096, seed=2).numpy(), tile]))
     st = _check(q, k, v, w.topk, "bf16", rows=rows, chunk=w.chunk)
+    print(f"long_65k: {st}")
     assert st["rows"] == len(rows)
+    assert st["exact_set_frac"] >= EXACT_FLOOR["long_65k"]
 
 
 def test_causal_16k_sampled_rows():
     w, (q, k, v) = _workload("causal_16k")
     L = w.Lq
+    heads = w.B * w.H
     first = np.arange(0, 200)  # rows i < k keep exactly {0..i}
-    pick = W.sample_rows(w.rows, 48, seed=3).numpy()
-    rows = np.unique(np.concatenate([first, L * 17 + first[:40], pick]))
+    # every row of one diagonal 128-query tile per head (a different tile for each head), the last 128
+    # rows of the last head, and 512 seeded rows
+    diag = np.concatenate([h * L + 128 * ((37 * h + 5) % (L // 128)) + np.arange(128) for h in range(heads)])
+    last = heads * L - 128 + np.arange(128)
+    pick = W.sample_rows(w.rows, 512, seed=3).numpy()
+    rows = np.unique(np.concatenate([first, diag, last, pick]))
     out, idx, score = _run(q, k, v, w.topk, w.chunk, causal=True)
-    check_rows(q=q, k=k, v=v, rows=rows, gpu_out=out[rows].numpy(), gpu_idx=idx[rows].numpy(),
-               gpu_score=score[rows].numpy(), topk=w.topk, dtype="bf16", causal=True)
+    st = check_rows(q=q, k=k, v=v, rows=rows, gpu_out=out[rows].numpy(), gpu_idx=idx[rows].numpy(),
+                    gpu_score=score[rows].numpy(), topk=w.topk, dtype="bf16", causal=True)
+    print(f"causal_16k: {st}")
+    assert st["rows"] >= 2048
+    assert st["exact_set_frac"] >= EXACT_FLOOR["causal_16k"]
     for i in range(w.topk):
         got = idx[i].numpy()
         assert sorted(got[got >= 0].tolist()) == list(range(i + 1))
@@ -161,28 +181,36 @@ def test_e2e_host_entry_in_head_slices_matches_device_entry(B, H, L, causal):
 
 
 def test_memory_is_linear_in_keys():
-    # Sec. 2.2: memory O(C L_K) for a fixed chunk; here the only device scratch is a fixed amount per
-    # CTA (the parked kept keys), the same for every L_K, so the peak is the inputs and outputs plus a
-    # constant: linear in L_K
-    peaks = []
-    for Lk in (8192, 16384, 32768, 65536):
-        q, k, v = W.attention_inputs(1, 4, 1024, Lk, 64, dtype="bf16", seed=Lk)
-        torch.cuda.synchronize()
-        torch.cuda.empty_cache()
-        torch.cuda.reset_peak_memory_stats()
-        base = torch.cuda.memory_allocated()
-        free0 = torch.cuda.mem_get_info()[0]
-        dq, dk, dv = q.cuda(), k.cuda(), v.cuda()
-        out = torch.empty_like(dq)
-        T.topk_attn_fwd(dq, dk, dv, out, 64, 1024)
+    # Sec. 2.2: memory O(C L_K) for a fixed chunk.  Measured at the long-sequence shape (H = 12,
+    # Lq = Lk up to 65536): the device memory of a call is its inputs and output, which the caller
+    # owns, plus what the library takes from its own pool, read here directly (high-water mark of the
+    # pool over the call).  The pool part must be the documented scratch, the same at every length, and
+    # no other device memory may appear during the call; the total is then linear in L_K.
+    peaks, pools = [], []
+    for L in (8192, 16384, 32768, 65536):
+        g = torch.Generator(device="cuda").manual_seed(L)
+        q, k, v = (torch.randn(1, 12, L, 64, generator=g, device="cuda").bfloat16() for _ in range(3))
+        out = torch.empty_like(q)
+        T.topk_attn_fwd(q, k, v, out, 64, 1024)  # warm: the pool reserves the scratch once
         T.topk_check()
-        peaks.append(torch.cuda.max_memory_allocated() - base)
-        assert torch.cuda.mem_get_info()[0] >= free0 - (dq.numel() * 2 * 4 + (64 << 20))
-        assert T.topk_attn_workspace_bytes(1, 4, 1024, Lk, 64, 64, 1024, 1) == T.topk_attn_workspace_bytes(
-            1, 4, 1024, 8192, 64, 64, 1024, 1)
-        del dq, dk, dv, out
+        torch.cuda.synchronize()
+        T.topk_pool_usage(reset_high=True)
+        free0 = torch.cuda.mem_get_info()[0]
+        T.topk_attn_fwd(q, k, v, out, 64, 1024)
+        T.topk_check()
+        torch.cuda.synchronize()
+        used_high, reserved = T.topk_pool_usage()
+        ws = T.topk_attn_workspace_bytes(1, 12, L, L, 64, 64, 1024, 1)
+        assert ws <= used_high <= ws + (2 << 20), (L, used_high, ws)
+        assert torch.cuda.mem_get_info()[0] >= free0  # nothing mapped outside the pool during the call
+        tensors = sum(t.numel() * t.element_size() for t in (q, k, v, out))
+        peaks.append(tensors + used_high)
+        pools.append(used_high)
+        del q, k, v, out
+    assert len(set(pools)) == 1, pools  # the library's scratch does not depend on L_K
     d = np.diff(peaks)
-    assert np.allclose(d[1:] / d[:-1], 2.0, rtol=0.02), peaks
+    assert np.allclose(d[1:] / d[:-1], 2.0, rtol=1e-9), peaks  # total = a * L_K + b
+    T.topk_pool_trim()
 
 
 def _exact_selection(q, k, v, topk, causal=False, rows=None):
