@@ -272,3 +272,11 @@ def test_two_level_heap_sizes(d, topk):
 def test_two_level_heap_exact_ties():
     q, k, v = W.attention_inputs(1, 2, 256, 8192, 64, dtype="bf16", seed=510, dist="integer")
     _exact_selection(q, k, v, 100)
+
+
+@pytest.mark.parametrize("d,topk", [(64, 1), (64, 17), (64, 64), (64, 100), (64, 128), (128, 5), (128, 64)])
+def test_ragged_long_rows(d, topk):
+    # long rows: a key count that is not a multiple of the key tile, query rows past the last full
+    # 128-row tile, several heads
+    q, k, v = W.attention_inputs(1, 3, 300, 33000 + d, d, dtype="bf16", seed=600 + topk + d)
+    _check(q, k, v, topk, "bf16")
