@@ -170,22 +170,37 @@ struct RowCand {
       hist_on = true;
       return;
     }
+    // scan from the top bin down, eight bins per step: the eight loads are
+    // independent, so their latencies overlap
     uint32_t acc = 0;
     int bstar = 0, bpart = -1;
-    for (int b = NBINS - 1; b >= 0; --b) {
-      acc += hist[b * BM];
-      if (bpart < 0 && acc >= static_cast<uint32_t>(kp)) bpart = b;  // kp <= k: found first
-      if (acc >= static_cast<uint32_t>(k)) {
-        bstar = b;
-        break;
+    for (int b0 = NBINS - 8; b0 >= 0; b0 -= 8) {
+      uint32_t h8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) h8[i] = hist[(b0 + i) * BM];
+      bool done = false;
+#pragma unroll
+      for (int i = 7; i >= 0; --i) {
+        if (done) continue;
+        acc += h8[i];
+        if (bpart < 0 && acc >= static_cast<uint32_t>(kp)) bpart = b0 + i;  // kp <= k: found first
+        if (acc >= static_cast<uint32_t>(k)) {
+          bstar = b0 + i;
+          done = true;
+        }
       }
+      if (done) break;
     }
     if (bpart >= 2) Lp = fmaxf(Lp, base + static_cast<float>(bpart - 1) * width);
     if (bstar >= 2) {
       L = fmaxf(L, base + static_cast<float>(bstar - 1) * width);
-      if (bstar >= NBINS / 2) {  // slide the window up
+      if (bstar >= NBINS / 2) {  // slide the window up: read every bin, then write
         const int sh = bstar - 1;
-        for (int b = 0; b < NBINS; ++b) hist[b * BM] = b + sh < NBINS ? hist[(b + sh) * BM] : 0u;
+        uint32_t h[NBINS];
+#pragma unroll
+        for (int b = 0; b < NBINS; ++b) h[b] = b + sh < NBINS ? hist[(b + sh) * BM] : 0u;
+#pragma unroll
+        for (int b = 0; b < NBINS; ++b) hist[b * BM] = h[b];
         base += static_cast<float>(sh) * width;
       }
     }
