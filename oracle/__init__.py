@@ -14,7 +14,10 @@ computes the paper's definitions directly:
 * Eq. 1 / Eq. 2 -- plain (optionally causal) attention over every key, the
   special case top-k reduces to when k equals the number of keys;
 * index-evaluate mode: the same activation and weighted sum for a given
-  kept set (used where the near-tie rule lets two correct sets differ).
+  kept set (used where the near-tie rule lets two correct sets differ);
+* the backward pass for a given kept set (Sec. 2.2): gradients with respect
+  to Q, K, V (x, W1, W2 for the feed-forward layer), the kept set being the
+  forward pass's cache.
 
 Ties are broken toward the lower key index; causal rows with fewer than k
 valid keys keep all of them.
@@ -34,7 +37,7 @@ _LIB = os.path.join(_HERE, "liboracle.so")
 _lock = threading.Lock()
 _lib = None
 
-F32, BF16 = 0, 1
+F32, BF16, F64 = 0, 1, 2
 SOFTMAX, RELU = 0, 1
 
 
@@ -63,8 +66,11 @@ def _load():
             lib.oracle_vanilla.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i32, vp, i64, vp, i32]
             lib.oracle_eval_indices.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i64, vp, i64,
                                                 vp, vp, vp, i32]
+            lib.oracle_topk_bwd.argtypes = [i32, i32, vp, vp, vp, i32, vp, i64, i64, i64, i64, i64, i64, vp,
+                                            vp, vp, vp, i32]
             lib.oracle_hardware_threads.argtypes = []
-            for f in (lib.oracle_topk, lib.oracle_vanilla, lib.oracle_eval_indices, lib.oracle_hardware_threads):
+            for f in (lib.oracle_topk, lib.oracle_vanilla, lib.oracle_eval_indices, lib.oracle_topk_bwd,
+                      lib.oracle_hardware_threads):
                 f.restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -75,7 +81,7 @@ def hardware_threads() -> int:
 
 
 def _as_raw(a):
-    """numpy float32 / uint16(bf16 bits) array, or a CPU torch tensor -> (contiguous ndarray, dtype code)."""
+    """numpy float32 / float64 / uint16(bf16 bits) array, or a CPU torch tensor -> (contiguous ndarray, dtype code)."""
     if not isinstance(a, np.ndarray):  # torch tensor
         import torch
 
@@ -84,13 +90,17 @@ def _as_raw(a):
             return t.view(torch.int16).numpy().view(np.uint16), BF16
         if t.dtype == torch.float32:
             return t.numpy(), F32
-        raise TypeError(f"oracle takes float32 or bfloat16, got {t.dtype}")
+        if t.dtype == torch.float64:
+            return t.numpy(), F64
+        raise TypeError(f"oracle takes float32, float64 or bfloat16, got {t.dtype}")
     a = np.ascontiguousarray(a)
     if a.dtype == np.float32:
         return a, F32
+    if a.dtype == np.float64:
+        return a, F64
     if a.dtype == np.uint16:
         return a, BF16
-    raise TypeError(f"oracle takes float32 or bf16-as-uint16 arrays, got {a.dtype}")
+    raise TypeError(f"oracle takes float32, float64 or bf16-as-uint16 arrays, got {a.dtype}")
 
 
 def _rows_arg(rows, total):
@@ -182,3 +192,37 @@ def ffn_dense(x, W1, W2, *, rows=None, threads: int = 0):
 def ffn_eval_indices(x, W1, W2, idx, *, rows=None, threads: int = 0):
     return eval_indices(x[None, None], W1[None, None], W2[None, None], idx, act=RELU, rows=rows,
                         threads=threads)
+
+
+def topk_attention_bwd(q, k, v, dout, idx, *, act: int = SOFTMAX, threads: int = 0):
+    """Backward pass of Eq. 4 (act=SOFTMAX) or Eq. 3 (act=RELU) for the kept sets idx.
+
+    q [B,H,Lq,d], k/v [B,H,Lk,d], dout [B,H,Lq,d] (any dtype the oracle reads), idx [B*H*Lq, topk]
+    int32 (-1 = empty slot).  Returns dict(dq [B,H,Lq,d], dk [B,H,Lk,d], dv [B,H,Lk,d]) in float64.
+    """
+    qa, ka, va, dt = _common(q, k, v, act)
+    ga, gdt = _as_raw(dout)
+    B, H, Lq, d = qa.shape
+    Lk = ka.shape[2]
+    if ka.shape != (B, H, Lk, d) or va.shape != (B, H, Lk, d) or ga.shape != (B, H, Lq, d):
+        raise ValueError("shape mismatch")
+    ia = np.ascontiguousarray(np.asarray(idx, dtype=np.int32))
+    if ia.ndim != 2 or ia.shape[0] != B * H * Lq:
+        raise ValueError("idx must be [B*H*Lq, topk]")
+    dq = np.zeros((B, H, Lq, d), np.float64)
+    dk = np.zeros((B, H, Lk, d), np.float64)
+    dv = np.zeros((B, H, Lk, d), np.float64)
+    rc = _load().oracle_topk_bwd(act, dt, qa.ctypes.data, ka.ctypes.data, va.ctypes.data, gdt, ga.ctypes.data,
+                                 B, H, Lq, Lk, d, ia.shape[1], ia.ctypes.data, dq.ctypes.data, dk.ctypes.data,
+                                 dv.ctypes.data, threads)
+    if rc:
+        raise RuntimeError(f"oracle_topk_bwd failed: {rc}")
+    return {"dq": dq, "dk": dk, "dv": dv}
+
+
+def ffn_bwd(x, W1, W2, dout, idx, *, threads: int = 0):
+    """Backward pass of the top-k feed-forward layer (Eq. 3): x [N,dm], W1/W2 [d_ff,dm], dout [N,dm],
+    idx [N, topk] -> dict(dx [N,dm], dW1 [d_ff,dm], dW2 [d_ff,dm]) in float64."""
+    g = topk_attention_bwd(x[None, None], W1[None, None], W2[None, None], dout[None, None], idx, act=RELU,
+                           threads=threads)
+    return {"dx": g["dq"][0, 0], "dW1": g["dk"][0, 0], "dW2": g["dv"][0, 0]}

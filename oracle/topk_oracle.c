@@ -27,7 +27,8 @@
  *   - top-k runs on the signed scores; ReLU is applied after selection.
  *
  * Arithmetic: inputs are widened exactly to double (bf16 by a 16-bit
- * shift); all sums, the softmax and the weighted sum are in double.
+ * shift; fp64 inputs, used by the finite-difference pins, are taken as
+ * they are); all sums, the softmax and the weighted sum are in double.
  * Selection keeps a bounded heap of the k+1 best entries so that the
  * (k+1)-th score, which decides the near-tie rule, is reported too.
  */
@@ -40,11 +41,13 @@
 
 #define ORACLE_F32 0
 #define ORACLE_BF16 1
+#define ORACLE_F64 2
 #define ACT_SOFTMAX 0
 #define ACT_RELU 1
 
 static double widen(const void* base, size_t i, int dtype) {
   if (dtype == ORACLE_F32) return (double)((const float*)base)[i];
+  if (dtype == ORACLE_F64) return ((const double*)base)[i];
   uint32_t bits = ((uint32_t)((const uint16_t*)base)[i]) << 16;
   float f;
   memcpy(&f, &bits, sizeof f);
@@ -329,6 +332,225 @@ int oracle_eval_indices(int act, int dtype, const void* q, const void* k, const 
   J.out = out;
   J.score = score;
   return run(J, nthreads);
+}
+
+/* ------------------------------------------------------------------------
+ * Backward pass for a given kept set (Sec. 2.2, "Improving efficiency
+ * through top-k attention").  The kept set of every row is the cache the
+ * forward pass leaves behind; the selection is piecewise constant in the
+ * scores, so the gradient reaches Q and K only through the kept scores.
+ * With L = sum_i dout_i . out_i, per row i (problem b, h) with kept keys
+ * j_1 .. j_n (idx entries < 0 are empty):
+ *
+ *   s_t   = q_i . k_{j_t}                    recomputed in double
+ *   a_t   = act(s)_t                          softmax over the kept entries
+ *                                             (Eq. 4) or ReLU (Eq. 3)
+ *   da_t  = dout_i . v_{j_t}                  dL/da_t
+ *   ds_t  = a_t (da_t - sum_u a_u da_u)       softmax
+ *         = da_t if s_t > 0, else 0           ReLU (derivative 0 at s = 0)
+ *   dq_i  = sum_t ds_t k_{j_t}
+ *   dk_j  = sum over (i, t) with j_t = j of ds_t q_i
+ *   dv_j  = sum over (i, t) with j_t = j of a_t dout_i
+ *
+ * Phase 1 runs the per-row steps (threads split the rows) and keeps a_t and
+ * ds_t; phase 2 forms dk and dv as the two sparse-by-dense products (threads
+ * split the keys of each problem into ranges; each key's terms are added in
+ * ascending (i, t) order).
+ * ---------------------------------------------------------------------- */
+typedef struct {
+  int act, dtype, dout_dtype;
+  const void *q, *k, *v, *dout;
+  int64_t Lq, Lk, d, topk;
+  const int32_t* idx;
+  double *a, *ds, *dq, *dk, *dv;
+  int64_t nchunk;     /* key ranges per problem (phase 2) */
+  int64_t begin, end; /* rows (phase 1) or (problem, key range) units (phase 2) */
+  int status;
+} bwd_job;
+
+static void* bwd_rows(void* arg) {
+  bwd_job* J = (bwd_job*)arg;
+  const int64_t d = J->d, K = J->topk;
+  double* qbuf = (double*)malloc(sizeof(double) * (size_t)d);
+  double* gbuf = (double*)malloc(sizeof(double) * (size_t)d);
+  double* s = (double*)malloc(sizeof(double) * (size_t)K);
+  double* da = (double*)malloc(sizeof(double) * (size_t)K);
+  if (!qbuf || !gbuf || !s || !da) {
+    J->status = -1;
+    goto done;
+  }
+  for (int64_t row = J->begin; row < J->end; ++row) {
+    const int64_t bh = row / J->Lq;
+    const int32_t* kept = J->idx + row * K;
+    double* a = J->a + row * K;
+    double* ds = J->ds + row * K;
+    for (int64_t c = 0; c < d; ++c) {
+      qbuf[c] = widen(J->q, (size_t)(row * d + c), J->dtype);
+      gbuf[c] = widen(J->dout, (size_t)(row * d + c), J->dout_dtype);
+    }
+    /* scores of the kept entries, and dL/da_t */
+    for (int64_t t = 0; t < K; ++t) {
+      s[t] = 0.0;
+      da[t] = 0.0;
+      a[t] = 0.0;
+      ds[t] = 0.0;
+      const int32_t j = kept[t];
+      if (j < 0) continue;
+      if (j >= J->Lk) {
+        J->status = -3;
+        continue;
+      }
+      const int64_t krow = bh * J->Lk + j;
+      for (int64_t c = 0; c < d; ++c) {
+        s[t] += qbuf[c] * widen(J->k, (size_t)(krow * d + c), J->dtype);
+        da[t] += gbuf[c] * widen(J->v, (size_t)(krow * d + c), J->dtype);
+      }
+    }
+    /* activation over the kept entries, then its backward */
+    if (J->act == ACT_SOFTMAX) {
+      double m = -INFINITY, z = 0.0, dot = 0.0;
+      for (int64_t t = 0; t < K; ++t)
+        if (kept[t] >= 0 && kept[t] < J->Lk && s[t] > m) m = s[t];
+      for (int64_t t = 0; t < K; ++t)
+        if (kept[t] >= 0 && kept[t] < J->Lk) {
+          a[t] = exp(s[t] - m);
+          z += a[t];
+        }
+      for (int64_t t = 0; t < K; ++t)
+        if (kept[t] >= 0 && kept[t] < J->Lk) {
+          a[t] /= z;
+          dot += a[t] * da[t];
+        }
+      for (int64_t t = 0; t < K; ++t)
+        if (kept[t] >= 0 && kept[t] < J->Lk) ds[t] = a[t] * (da[t] - dot);
+    } else {
+      for (int64_t t = 0; t < K; ++t)
+        if (kept[t] >= 0 && kept[t] < J->Lk) {
+          a[t] = s[t] > 0.0 ? s[t] : 0.0;
+          ds[t] = s[t] > 0.0 ? da[t] : 0.0;
+        }
+    }
+    /* dq_i = sum_t ds_t k_{j_t} */
+    double* dq = J->dq + row * d;
+    for (int64_t c = 0; c < d; ++c) dq[c] = 0.0;
+    for (int64_t t = 0; t < K; ++t) {
+      const int32_t j = kept[t];
+      if (j < 0 || j >= J->Lk) continue;
+      const int64_t krow = bh * J->Lk + j;
+      for (int64_t c = 0; c < d; ++c) dq[c] += ds[t] * widen(J->k, (size_t)(krow * d + c), J->dtype);
+    }
+  }
+done:
+  free(qbuf);
+  free(gbuf);
+  free(s);
+  free(da);
+  return NULL;
+}
+
+/* Phase 2: the units [begin, end) are (problem, key range) pairs, nchunk
+ * ranges per problem.  A unit scans its problem's kept sets in ascending
+ * (i, t) order and adds each term whose key falls in its range. */
+static void* bwd_keys(void* arg) {
+  bwd_job* J = (bwd_job*)arg;
+  const int64_t d = J->d, K = J->topk, C = J->nchunk;
+  for (int64_t u = J->begin; u < J->end; ++u) {
+    const int64_t bh = u / C, c = u % C;
+    const int64_t j0 = c * J->Lk / C, j1 = (c + 1) * J->Lk / C;
+    for (int64_t j = j0; j < j1; ++j)
+      for (int64_t e = 0; e < d; ++e) {
+        J->dk[(bh * J->Lk + j) * d + e] = 0.0;
+        J->dv[(bh * J->Lk + j) * d + e] = 0.0;
+      }
+    for (int64_t i = 0; i < J->Lq; ++i) {
+      const int64_t row = bh * J->Lq + i;
+      const int32_t* kept = J->idx + row * K;
+      for (int64_t t = 0; t < K; ++t) {
+        const int64_t j = kept[t];
+        if (j < j0 || j >= j1) continue;
+        const double a = J->a[row * K + t], g = J->ds[row * K + t];
+        double* dk = J->dk + (bh * J->Lk + j) * d;
+        double* dv = J->dv + (bh * J->Lk + j) * d;
+        for (int64_t e = 0; e < d; ++e) {
+          dk[e] += g * widen(J->q, (size_t)(row * d + e), J->dtype);
+          dv[e] += a * widen(J->dout, (size_t)(row * d + e), J->dout_dtype);
+        }
+      }
+    }
+  }
+  return NULL;
+}
+
+static int bwd_run(bwd_job proto, int64_t total, int phase, int nthreads) {
+  if (nthreads <= 0) nthreads = (int)sysconf(_SC_NPROCESSORS_ONLN);
+  if (nthreads < 1) nthreads = 1;
+  if (nthreads > total) nthreads = (int)(total > 0 ? total : 1);
+  bwd_job* jobs = (bwd_job*)calloc((size_t)nthreads, sizeof(bwd_job));
+  pthread_t* th = (pthread_t*)calloc((size_t)nthreads, sizeof(pthread_t));
+  if (!jobs || !th) {
+    free(jobs);
+    free(th);
+    return -1;
+  }
+  const int64_t per = (total + nthreads - 1) / nthreads;
+  for (int t = 0; t < nthreads; ++t) {
+    jobs[t] = proto;
+    jobs[t].begin = (int64_t)t * per < total ? (int64_t)t * per : total;
+    jobs[t].end = jobs[t].begin + per < total ? jobs[t].begin + per : total;
+    jobs[t].status = 0;
+    pthread_create(&th[t], NULL, phase == 1 ? bwd_rows : bwd_keys, &jobs[t]);
+  }
+  int status = 0;
+  for (int t = 0; t < nthreads; ++t) {
+    pthread_join(th[t], NULL);
+    if (jobs[t].status) status = jobs[t].status;
+  }
+  free(jobs);
+  free(th);
+  return status;
+}
+
+/* Gradients of Eq. 4 (act = ACT_SOFTMAX) or Eq. 3 (act = ACT_RELU, with
+ * B = H = 1: q = x, k = W1, v = W2) with respect to q, k and v, for the
+ * kept sets idx [B*H*Lq][topk] (-1 = empty slot) and the output gradient
+ * dout [B*H*Lq][d] (its own dtype code).  Outputs, all rows: dq
+ * [B*H*Lq][d], dk and dv [B*H*Lk][d].  Every kept index must be < Lk
+ * (-3 otherwise). */
+int oracle_topk_bwd(int act, int dtype, const void* q, const void* k, const void* v, int dout_dtype,
+                    const void* dout, int64_t B, int64_t H, int64_t Lq, int64_t Lk, int64_t d,
+                    int64_t topk, const int32_t* idx, double* dq, double* dk, double* dv, int nthreads) {
+  if (d <= 0 || Lq <= 0 || Lk <= 0 || topk < 1 || B <= 0 || H <= 0) return -2;
+  bwd_job J;
+  memset(&J, 0, sizeof J);
+  J.act = act;
+  J.dtype = dtype;
+  J.dout_dtype = dout_dtype;
+  J.q = q;
+  J.k = k;
+  J.v = v;
+  J.dout = dout;
+  J.Lq = Lq;
+  J.Lk = Lk;
+  J.d = d;
+  J.topk = topk;
+  J.idx = idx;
+  J.dq = dq;
+  J.dk = dk;
+  J.dv = dv;
+  const int64_t rows = B * H * Lq;
+  J.a = (double*)malloc(sizeof(double) * (size_t)(rows * topk));
+  J.ds = (double*)malloc(sizeof(double) * (size_t)(rows * topk));
+  int rc = -1;
+  if (J.a && J.ds) {
+    int nt = nthreads > 0 ? nthreads : (int)sysconf(_SC_NPROCESSORS_ONLN);
+    if (nt < 1) nt = 1;
+    J.nchunk = nt < Lk ? nt : Lk;
+    rc = bwd_run(J, rows, 1, nt);
+    if (rc == 0) rc = bwd_run(J, B * H * J.nchunk, 2, nt);
+  }
+  free(J.a);
+  free(J.ds);
+  return rc;
 }
 
 int oracle_hardware_threads(void) { return (int)sysconf(_SC_NPROCESSORS_ONLN); }
