@@ -13,6 +13,11 @@
  *                     out = sum over the k largest s_j = x . W1_j of
  *                     ReLU(s_j) * W2_j.  Keys and values are the ROWS of W1
  *                     and W2.
+ *   topk_attn_bwd  -- the backward pass of Eq. 4 for the kept set the forward
+ *   topk_ffn_bwd      pass cached (Sec. 2.2 "Improving efficiency through
+ *                     top-k attention"): gradients of q, k, v (x, W1, W2)
+ *                     from dout, the kept indices and their scores, with the
+ *                     activation recomputed from the cached scores.
  * Query chunking (Sec. 2.2 "Query chunking") bounds scheduling only: results
  * never depend on `chunk`, and no [chunk x L_K] score matrix is ever stored
  * in device memory.
@@ -123,6 +128,57 @@ int topk_ffn_fwd(const void* x, const void* W1, const void* W2, void* out, int N
 /* topk_ffn_fwd plus the kept indices [N, topk] int32 and scores [N, topk] fp32. */
 int topk_ffn_fwd_indices(const void* x, const void* W1, const void* W2, void* out, int N, int d_model,
                          int d_ff, int topk, int32_t* idx, float* score, void* stream);
+
+/*
+ * Backward pass of top-k attention (Sec. 2.2, "Improving efficiency through
+ * top-k attention"): the forward pass caches, per query row, the kept key
+ * indices and their scores (topk_attn_fwd_indices writes exactly that
+ * cache), and the backward pass recomputes only the activation over them.
+ * With L = sum over rows of dout_i . out_i and the kept set held fixed:
+ *   a_t  = softmax over the row's kept scores,  da_t = dout_i . v_{j_t},
+ *   ds_t = a_t (da_t - sum_u a_u da_u),
+ *   dq_i = sum_t ds_t k_{j_t};  dk_j, dv_j = the sums of ds_t q_i and
+ *   a_t dout_i over every (i, t) that kept key j of the same (b, h).
+ *   q, k, v : the forward pass's inputs (device, `dtype`, layouts above).
+ *   dout    : [B, H, Lq, d] device, `dtype` (the dtype of out).
+ *   idx     : [B, H, Lq, topk] int32 device, the cached kept indices; an entry
+ *             outside [0, Lk) (the forward pass pads with -1) is an empty slot.
+ *   score   : [B, H, Lq, topk] fp32 device, the cached scores s_t = q_i . k_{j_t}.
+ *   dq      : [B, H, Lq, d] fp32 device (written).
+ *   dk, dv  : [B, H, Lk, d] fp32 device (written; keys no row kept get 0).
+ *   d       : TOPK_BF16: 64 or 128.  TOPK_F32: 16, 32, 64 or 128.
+ *   topk    : the cache's width, 1 <= topk <= 2048.  B*H*Lq*topk and B*H*Lk
+ *             must stay below 2^31.
+ *   Any order of the kept entries within a row gives the same result.  dk and
+ *   dv add each key's terms in an order that depends on atomic ranks, so
+ *   they can differ in the last bits from call to call.
+ *   Scratch: topk_attn_bwd_workspace_bytes() (20 bytes per cache entry plus
+ *   8 bytes per key), from the library's pool.  Errors as topk_attn_fwd.
+ */
+int topk_attn_bwd(const void* q, const void* k, const void* v, const void* dout, const int32_t* idx,
+                  const float* score, float* dq, float* dk, float* dv, int B, int H, int Lq, int Lk, int d,
+                  int topk, int dtype, void* stream);
+
+/*
+ * Backward pass of the top-k feed-forward layer (Eq. 3 with ReLU, Sec. 2.1
+ * and Sec. 2.2) for the cache of topk_ffn_fwd_indices:
+ *   a_t = ReLU(s_t),  ds_t = (dout_i . W2_{j_t}) if s_t > 0 else 0,
+ *   dx_i = sum_t ds_t W1_{j_t};  dW1_j, dW2_j = the sums of ds_t x_i and
+ *   a_t dout_i over every (i, t) that kept key j.
+ *   x, W1, W2 : the forward pass's inputs (bf16 device, layouts above).
+ *   dout      : [N, d_model] fp32 device (the dtype of the forward output).
+ *   idx, score: [N, topk] int32 / fp32 device, the cache.
+ *   dx        : [N, d_model] fp32; dW1, dW2: [d_ff, d_model] fp32 (written).
+ *   d_model   : a multiple of 64, at most 2048.  1 <= topk <= d_ff.
+ *   Scratch: topk_ffn_bwd_workspace_bytes().  Errors as topk_ffn_fwd.
+ */
+int topk_ffn_bwd(const void* x, const void* W1, const void* W2, const float* dout, const int32_t* idx,
+                 const float* score, float* dx, float* dW1, float* dW2, int N, int d_model, int d_ff, int topk,
+                 void* stream);
+
+/* Scratch bytes of the two backward calls for these arguments; 0 if invalid or unsupported. */
+size_t topk_attn_bwd_workspace_bytes(int B, int H, int Lq, int Lk, int d, int topk, int dtype);
+size_t topk_ffn_bwd_workspace_bytes(int N, int d_model, int d_ff, int topk);
 
 /*
  * topk_ffn_fwd without any device allocation.  The paper has no counterpart:

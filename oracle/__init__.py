@@ -65,7 +65,7 @@ def _load():
                                         vp, vp, vp, vp, i32]
             lib.oracle_vanilla.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i32, vp, i64, vp, i32]
             lib.oracle_eval_indices.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i64, vp, i64,
-                                                vp, vp, vp, i32]
+                                                vp, vp, vp, vp, i32]
             lib.oracle_topk_bwd.argtypes = [i32, i32, vp, vp, vp, i32, vp, i64, i64, i64, i64, i64, i64, vp,
                                             vp, vp, vp, i32]
             lib.oracle_hardware_threads.argtypes = []
@@ -159,8 +159,11 @@ def vanilla(q, k, v, *, act: int = SOFTMAX, causal: bool = False, rows=None, thr
     return out
 
 
-def eval_indices(q, k, v, idx, *, act: int = SOFTMAX, rows=None, threads: int = 0):
-    """Index-evaluate: given kept sets idx [n, topk] (-1 = empty), return (out [n,d], score [n,topk])."""
+def eval_indices(q, k, v, idx, *, act: int = SOFTMAX, rows=None, threads: int = 0, return_idx: bool = False):
+    """Index-evaluate: given kept sets idx [n, topk] (-1 = empty), return (out [n,d], score [n,topk]).
+
+    score lists each row's kept entries in the total order (score descending, index
+    ascending), -inf padded; with return_idx the matching indices (-1 padded) come third."""
     qa, ka, va, dt = _common(q, k, v, act)
     B, H, Lq, d = qa.shape
     Lk = ka.shape[2]
@@ -171,11 +174,13 @@ def eval_indices(q, k, v, idx, *, act: int = SOFTMAX, rows=None, threads: int = 
     K = ia.shape[1]
     out = np.zeros((n, d), np.float64)
     score = np.zeros((n, K), np.float64)
+    iout = np.zeros((n, K), np.int32) if return_idx else None
     rc = _load().oracle_eval_indices(act, dt, qa.ctypes.data, ka.ctypes.data, va.ctypes.data, B, H, Lq, Lk, d,
-                                     K, rp, n, ia.ctypes.data, out.ctypes.data, score.ctypes.data, threads)
+                                     K, rp, n, ia.ctypes.data, out.ctypes.data, score.ctypes.data,
+                                     None if iout is None else iout.ctypes.data, threads)
     if rc:
         raise RuntimeError(f"oracle_eval_indices failed: {rc}")
-    return out, score
+    return (out, score, iout) if return_idx else (out, score)
 
 
 def ffn(x, W1, W2, topk: int, *, rows=None, threads: int = 0):

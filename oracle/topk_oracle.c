@@ -309,11 +309,13 @@ int oracle_vanilla(int act, int dtype, const void* q, const void* k, const void*
 
 /* Index-evaluate: the kept set of each listed row is given in idx
  * ([nrows][topk], -1 = empty slot); scores are recomputed in double and
- * the activation and weighted sum follow Eq. 4 / Eq. 3 from there. */
+ * the activation and weighted sum follow Eq. 4 / Eq. 3 from there.  score
+ * and, if idx_out is not NULL, idx_out receive the kept entries in the
+ * total order (score descending, index ascending), padded with -inf / -1. */
 int oracle_eval_indices(int act, int dtype, const void* q, const void* k, const void* v, int64_t B,
                         int64_t H, int64_t Lq, int64_t Lk, int64_t d, int64_t topk,
                         const int64_t* rows, int64_t nrows, const int32_t* idx, double* out,
-                        double* score, int nthreads) {
+                        double* score, int32_t* idx_out, int nthreads) {
   job J;
   memset(&J, 0, sizeof J);
   J.act = act;
@@ -331,6 +333,7 @@ int oracle_eval_indices(int act, int dtype, const void* q, const void* k, const 
   J.eval_idx = idx;
   J.out = out;
   J.score = score;
+  J.idx = idx_out;
   return run(J, nthreads);
 }
 

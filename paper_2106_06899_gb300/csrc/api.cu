@@ -177,6 +177,58 @@ int run_ffn(FfnArgs a, cudaStream_t st) {
 
 size_t elem_bytes(int dtype) { return dtype == TOPK_F32 ? 4 : 2; }
 
+// Backward pass (bwd.cu): the cache width, the entry and bucket counts are
+// bounded so that slots and offsets fit in 32-bit integers.
+constexpr int kBwdMaxK = 2048;
+
+int validate_attn_bwd(const AttnBwdArgs& a) {
+  if (!a.q || !a.k || !a.v || !a.dout || !a.idx || !a.score || !a.dq || !a.dk || !a.dv) return TOPK_ERR_INVALID_ARG;
+  if (a.B <= 0 || a.H <= 0 || a.Lq <= 0 || a.Lk <= 0 || a.d <= 0) return TOPK_ERR_INVALID_ARG;
+  if (a.topk < 1 || a.topk > a.Lk) return TOPK_ERR_INVALID_ARG;
+  if (a.dtype != TOPK_F32 && a.dtype != TOPK_BF16) return TOPK_ERR_INVALID_ARG;
+  if (a.topk > kBwdMaxK || !attn_bwd_supports(a.d, a.dtype)) return TOPK_ERR_UNSUPPORTED;
+  const long long BH = static_cast<long long>(a.B) * a.H;
+  if (BH * a.Lq * a.topk >= (1ll << 31) || BH * a.Lk >= (1ll << 31)) return TOPK_ERR_UNSUPPORTED;
+  for (const void* p : {a.q, a.k, a.v, a.dout, static_cast<const void*>(a.dq), static_cast<const void*>(a.dk),
+                        static_cast<const void*>(a.dv)})
+    if (!aligned16(p)) return TOPK_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(a.idx) & 3u) || (reinterpret_cast<uintptr_t>(a.score) & 3u))
+    return TOPK_ERR_UNSUPPORTED;
+  return TOPK_OK;
+}
+
+int validate_ffn_bwd(const FfnBwdArgs& a) {
+  if (!a.x || !a.W1 || !a.W2 || !a.dout || !a.idx || !a.score || !a.dx || !a.dW1 || !a.dW2)
+    return TOPK_ERR_INVALID_ARG;
+  if (a.N <= 0 || a.d_model <= 0 || a.d_ff <= 0) return TOPK_ERR_INVALID_ARG;
+  if (a.topk < 1 || a.topk > a.d_ff) return TOPK_ERR_INVALID_ARG;
+  if (a.d_model % 64 != 0 || a.d_model > 2048) return TOPK_ERR_UNSUPPORTED;
+  if (static_cast<long long>(a.N) * a.topk >= (1ll << 31)) return TOPK_ERR_UNSUPPORTED;
+  for (const void* p : {a.x, a.W1, a.W2, static_cast<const void*>(a.dout), static_cast<const void*>(a.dx),
+                        static_cast<const void*>(a.dW1), static_cast<const void*>(a.dW2)})
+    if (!aligned16(p)) return TOPK_ERR_UNSUPPORTED;
+  if ((reinterpret_cast<uintptr_t>(a.idx) & 3u) || (reinterpret_cast<uintptr_t>(a.score) & 3u))
+    return TOPK_ERR_UNSUPPORTED;
+  return TOPK_OK;
+}
+
+template <typename Args, typename Size, typename Run>
+int run_bwd(Args a, int rc, Size size, Run launch, cudaStream_t st) {
+  if (rc) return rc;
+  DeviceState* dev = device_state();
+  if (!dev) return TOPK_ERR_NO_DEVICE;
+  if (dev->cc_major != 10 || dev->cc_minor != 3) return TOPK_ERR_NO_DEVICE;
+  void* buf = nullptr;
+  if (!pool_alloc(&buf, size(a), st)) return TOPK_ERR_CUDA;
+  a.workspace = buf;
+  const int n = launch(a, dev->num_sms, st);
+  cudaFreeAsync(buf, st);
+  if (n == 0) return TOPK_ERR_UNSUPPORTED;
+  if (n < 0) return TOPK_ERR_CUDA;
+  t_last_launches = n;
+  return TOPK_OK;
+}
+
 }  // namespace
 
 EncodeTiledFn encode_tiled_fn() {
@@ -236,6 +288,43 @@ int topk_ffn_fwd_indices(const void* x, const void* W1, const void* W2, void* ou
                          int topk, int32_t* idx, float* score, void* stream) {
   FfnArgs a{x, W1, W2, static_cast<float*>(out), N, d_model, d_ff, topk, idx, score, nullptr, 0};
   return run_ffn(a, static_cast<cudaStream_t>(stream));
+}
+
+int topk_attn_bwd(const void* q, const void* k, const void* v, const void* dout, const int32_t* idx,
+                  const float* score, float* dq, float* dk, float* dv, int B, int H, int Lq, int Lk, int d,
+                  int topk, int dtype, void* stream) {
+  AttnBwdArgs a{q, k, v, dout, idx, score, dq, dk, dv, B, H, Lq, Lk, d, topk, dtype, nullptr};
+  return run_bwd(
+      a, validate_attn_bwd(a),
+      [](const AttnBwdArgs& x) { return attn_bwd_workspace_bytes(x.B, x.H, x.Lq, x.Lk, x.topk); },
+      [](const AttnBwdArgs& x, int sms, cudaStream_t s) { return attn_bwd(x, sms, s); },
+      static_cast<cudaStream_t>(stream));
+}
+
+int topk_ffn_bwd(const void* x, const void* W1, const void* W2, const float* dout, const int32_t* idx,
+                 const float* score, float* dx, float* dW1, float* dW2, int N, int d_model, int d_ff, int topk,
+                 void* stream) {
+  FfnBwdArgs a{x, W1, W2, dout, idx, score, dx, dW1, dW2, N, d_model, d_ff, topk, nullptr};
+  return run_bwd(
+      a, validate_ffn_bwd(a), [](const FfnBwdArgs& y) { return ffn_bwd_workspace_bytes(y.N, y.d_ff, y.topk); },
+      [](const FfnBwdArgs& y, int sms, cudaStream_t s) { return ffn_bwd(y, sms, s); },
+      static_cast<cudaStream_t>(stream));
+}
+
+size_t topk_attn_bwd_workspace_bytes(int B, int H, int Lq, int Lk, int d, int topk, int dtype) {
+  void* p = reinterpret_cast<void*>(16);
+  float* f = reinterpret_cast<float*>(16);
+  AttnBwdArgs a{p, p, p, p, reinterpret_cast<const int32_t*>(16), f, f, f, f, B, H, Lq, Lk, d, topk, dtype, nullptr};
+  if (validate_attn_bwd(a) != TOPK_OK) return 0;
+  return attn_bwd_workspace_bytes(B, H, Lq, Lk, topk);
+}
+
+size_t topk_ffn_bwd_workspace_bytes(int N, int d_model, int d_ff, int topk) {
+  void* p = reinterpret_cast<void*>(16);
+  float* f = reinterpret_cast<float*>(16);
+  FfnBwdArgs a{p, p, p, f, reinterpret_cast<const int32_t*>(16), f, f, f, f, N, d_model, d_ff, topk, nullptr};
+  if (validate_ffn_bwd(a) != TOPK_OK) return 0;
+  return ffn_bwd_workspace_bytes(N, d_ff, topk);
 }
 
 size_t topk_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, int topk, int chunk, int dtype) {

@@ -58,6 +58,43 @@ size_t attn_tc_workspace_bytes(const AttnArgs& a, int num_sms);
 size_t ffn_workspace_bytes(int N, int d_model, int d_ff, int topk);
 int ffn_tc(const FfnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st);
 
+// Backward pass for a cached kept set (bwd.cu).  idx/score are the forward
+// pass's [rows][topk] cache (-1 / -inf = empty slot); dq [rows][d], dk and dv
+// [B*H*Lk][d] are fp32; dout has the dtype of q (attention) or is fp32 (FF).
+struct AttnBwdArgs {
+  const void* q;
+  const void* k;
+  const void* v;
+  const void* dout;
+  const int32_t* idx;
+  const float* score;
+  float* dq;
+  float* dk;
+  float* dv;
+  int B, H, Lq, Lk, d, topk, dtype;
+  void* workspace;  // attn_bwd_workspace_bytes
+};
+
+struct FfnBwdArgs {
+  const void* x;
+  const void* W1;
+  const void* W2;
+  const float* dout;
+  const int32_t* idx;
+  const float* score;
+  float* dx;
+  float* dW1;
+  float* dW2;
+  int N, d_model, d_ff, topk;
+  void* workspace;  // ffn_bwd_workspace_bytes
+};
+
+size_t attn_bwd_workspace_bytes(int B, int H, int Lq, int Lk, int topk);
+size_t ffn_bwd_workspace_bytes(int N, int d_ff, int topk);
+bool attn_bwd_supports(int d, int dtype);
+int attn_bwd(const AttnBwdArgs& a, int num_sms, cudaStream_t st);
+int ffn_bwd(const FfnBwdArgs& a, int num_sms, cudaStream_t st);
+
 // Driver entry point for cuTensorMapEncodeTiled (resolved once, no libcuda link).
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                    const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,

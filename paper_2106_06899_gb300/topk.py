@@ -49,6 +49,12 @@ def lib() -> ctypes.CDLL:
             L.topk_attn_workspace_bytes.restype = sz
             L.topk_ffn_workspace_bytes.argtypes = [i32] * 4
             L.topk_ffn_workspace_bytes.restype = sz
+            L.topk_attn_bwd.argtypes = [vp] * 9 + [i32] * 7 + [vp]
+            L.topk_ffn_bwd.argtypes = [vp] * 9 + [i32] * 4 + [vp]
+            L.topk_attn_bwd_workspace_bytes.argtypes = [i32] * 7
+            L.topk_attn_bwd_workspace_bytes.restype = sz
+            L.topk_ffn_bwd_workspace_bytes.argtypes = [i32] * 4
+            L.topk_ffn_bwd_workspace_bytes.restype = sz
             L.topk_check.argtypes = [vp]
             L.topk_error_string.argtypes = [i32]
             L.topk_error_string.restype = ctypes.c_char_p
@@ -61,7 +67,8 @@ def lib() -> ctypes.CDLL:
             for f in ("topk_attn_fwd", "topk_attn_fwd_indices", "topk_ffn_fwd", "topk_ffn_fwd_indices",
                       "topk_attn_fwd_host", "topk_ffn_fwd_host", "topk_ffn_fwd_noalloc", "topk_check",
                       "topk_last_launch_count",
-                      "topk_debug_skip_arrive", "topk_pool_usage", "topk_pool_trim"):
+                      "topk_debug_skip_arrive", "topk_pool_usage", "topk_pool_trim", "topk_attn_bwd",
+                      "topk_ffn_bwd"):
                 getattr(L, f).restype = i32
             _lib = L
     return _lib
@@ -186,6 +193,47 @@ def topk_ffn_fwd_noalloc(x, W1, W2, out, topk: int, stream=None) -> None:
     _check(rc, "topk_ffn_fwd_noalloc")
 
 
+def _cache_check(idx, score, rows_shape, topk):
+    want = (*rows_shape, topk)
+    for name, t, dt in (("idx", idx, torch.int32), ("score", score, torch.float32)):
+        if t.dtype != dt or tuple(t.shape) != want or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous {list(want)} {dt} tensor")
+
+
+def topk_attn_bwd(q, k, v, dout, idx, score, dq, dk, dv, stream=None) -> None:
+    """Backward pass of Eq. 4 for the cached kept set (Sec. 2.2): fp32 dq [B,H,Lq,d], dk/dv [B,H,Lk,d]."""
+    B, H, Lq, Lk, d = _attn_dims(q, k, v, dout)
+    topk = idx.shape[-1]
+    _cache_check(idx, score, (B, H, Lq), topk)
+    for name, t, shape in (("dq", dq, (B, H, Lq, d)), ("dk", dk, (B, H, Lk, d)), ("dv", dv, (B, H, Lk, d))):
+        if t.dtype != torch.float32 or tuple(t.shape) != shape or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous {list(shape)} float32 tensor")
+    rc = lib().topk_attn_bwd(_ptr(q), _ptr(k), _ptr(v), _ptr(dout), _ptr(idx), _ptr(score), _ptr(dq), _ptr(dk),
+                             _ptr(dv), B, H, Lq, Lk, d, int(topk), _dtype_code(q), _stream(stream))
+    _check(rc, "topk_attn_bwd")
+
+
+def topk_ffn_bwd(x, W1, W2, dout, idx, score, dx, dW1, dW2, stream=None) -> None:
+    """Backward pass of the top-k FF layer (Eq. 3) for the cached kept set: fp32 dx, dW1, dW2."""
+    N, dm, dff = _ffn_dims(x, W1, W2, dout)
+    topk = idx.shape[-1]
+    _cache_check(idx, score, (N,), topk)
+    for name, t, shape in (("dx", dx, (N, dm)), ("dW1", dW1, (dff, dm)), ("dW2", dW2, (dff, dm))):
+        if t.dtype != torch.float32 or tuple(t.shape) != shape or not t.is_contiguous():
+            raise ValueError(f"{name} must be a contiguous {list(shape)} float32 tensor")
+    rc = lib().topk_ffn_bwd(_ptr(x), _ptr(W1), _ptr(W2), _ptr(dout), _ptr(idx), _ptr(score), _ptr(dx), _ptr(dW1),
+                            _ptr(dW2), N, dm, dff, int(topk), _stream(stream))
+    _check(rc, "topk_ffn_bwd")
+
+
+def topk_attn_bwd_workspace_bytes(B, H, Lq, Lk, d, topk, dtype) -> int:
+    return int(lib().topk_attn_bwd_workspace_bytes(B, H, Lq, Lk, d, topk, dtype))
+
+
+def topk_ffn_bwd_workspace_bytes(N, d_model, d_ff, topk) -> int:
+    return int(lib().topk_ffn_bwd_workspace_bytes(N, d_model, d_ff, topk))
+
+
 def topk_attn_workspace_bytes(B, H, Lq, Lk, d, topk, chunk, dtype) -> int:
     return int(lib().topk_attn_workspace_bytes(B, H, Lq, Lk, d, topk, chunk, dtype))
 
@@ -244,3 +292,22 @@ def ffn(x, W1, W2, topk: int, return_indices: bool = False, stream=None):
     score = torch.empty(x.shape[0], topk, dtype=torch.float32, device=x.device)
     topk_ffn_fwd_indices(x, W1, W2, out, topk, idx, score, stream)
     return out, idx, score
+
+
+def attention_bwd(q, k, v, dout, idx, score, stream=None):
+    """Gradients (dq, dk, dv), fp32, of top-k attention for the cache (idx, score) of attention(...,
+    return_indices=True)."""
+    dq = torch.empty(q.shape, dtype=torch.float32, device=q.device)
+    dk = torch.empty(k.shape, dtype=torch.float32, device=k.device)
+    dv = torch.empty(v.shape, dtype=torch.float32, device=v.device)
+    topk_attn_bwd(q, k, v, dout, idx, score, dq, dk, dv, stream)
+    return dq, dk, dv
+
+
+def ffn_bwd(x, W1, W2, dout, idx, score, stream=None):
+    """Gradients (dx, dW1, dW2), fp32, of the top-k FF layer for the cache of ffn(..., return_indices=True)."""
+    dx = torch.empty(x.shape, dtype=torch.float32, device=x.device)
+    dW1 = torch.empty(W1.shape, dtype=torch.float32, device=W1.device)
+    dW2 = torch.empty(W2.shape, dtype=torch.float32, device=W2.device)
+    topk_ffn_bwd(x, W1, W2, dout, idx, score, dx, dW1, dW2, stream)
+    return dx, dW1, dW2

@@ -152,3 +152,79 @@ def sample_rows(total: int, n: int, seed: int = 0) -> torch.Tensor:
     if n > 1:
         pick[1] = total - 1
     return torch.unique(pick).sort().values
+
+
+def grad_output(shape, *, dtype="bf16", seed=0) -> torch.Tensor:
+    """dL/dout for the backward pass: N(0, 1) entries in ``dtype`` ("f32" or "bf16")."""
+    g = torch.Generator().manual_seed(int(seed) + 777)
+    return torch.randn(*shape, generator=g).to(_torch_dtype(dtype)).contiguous()
+
+
+def kept_sets(problems: int, Lq: int, Lk: int, k: int, *, seed=0, hot: int = 0, hot_frac: float = 0.0,
+              causal: bool = False, empty_frac: float = 0.0) -> torch.Tensor:
+    """A kept-set cache [problems * Lq, k] int32 of distinct keys per row, -1 for empty slots.
+
+    Drawn at random, not selected by score: the backward pass is defined for any kept
+    set.  ``hot`` keys (0 .. hot-1) each enter a fraction ``hot_frac`` of the rows, so
+    a few keys are kept by many rows, as the largest keys of a low-rank input are.
+    With ``causal`` row i draws from keys 0 .. i only (all of them when i < k)."""
+    g = torch.Generator().manual_seed(int(seed) + 4242)
+    rows = problems * Lq
+    n_valid = torch.full((rows,), Lk, dtype=torch.int64)
+    if causal:
+        n_valid = torch.clamp(torch.arange(rows) % Lq + 1, max=Lk)
+    idx = torch.full((rows, k), -1, dtype=torch.int64)
+    if hot:
+        hot_in = torch.rand(rows, hot, generator=g) < hot_frac
+        hot_in &= torch.arange(hot)[None, :] < n_valid[:, None]
+    else:
+        hot_in = torch.zeros(rows, 0, dtype=torch.bool)
+    n_hot = hot_in.sum(1) if hot else torch.zeros(rows, dtype=torch.int64)
+    # rows with few valid keys: a full permutation of them
+    small = n_valid <= 4 * k
+    for r in torch.nonzero(small).flatten().tolist():
+        nv = int(n_valid[r])
+        perm = torch.randperm(nv, generator=g)
+        if hot:
+            first = torch.nonzero(hot_in[r]).flatten()
+            rest = perm[~torch.isin(perm, first)]
+            perm = torch.cat([first, rest])
+        take = min(k, nv)
+        idx[r, :take] = perm[:take]
+    # other rows: the hot keys they enter, then the rest of k from an arithmetic
+    # progression hot + (base + t * stride) mod m over the m = n_valid - hot other keys,
+    # with a random base and a random stride prime to m (so its first k terms differ)
+    big = torch.nonzero(~small).flatten()
+    if big.numel():
+        m = n_valid[big] - hot
+        base = (torch.rand(big.numel(), generator=g) * m).long()
+        stride = 1 + (torch.rand(big.numel(), generator=g) * (m - 1)).long()
+        bad = torch.gcd(stride, m) != 1
+        while bool(bad.any()):
+            stride = torch.where(bad, stride % (m - 1) + 1, stride)
+            bad = torch.gcd(stride, m) != 1
+        prog = torch.empty(big.numel(), k, dtype=torch.int64)
+        x = base.clone()
+        for t in range(k):  # x_t = (base + t stride) mod m, one add and one wrap per term
+            prog[:, t] = x
+            x += stride
+            x -= m * (x >= m)
+        prog += hot
+        if hot:
+            # the hot keys a row enters take its last slots
+            filled = torch.zeros(big.numel(), dtype=torch.int64)
+            hb = hot_in[big]
+            rows_b = torch.arange(big.numel())
+            for h in range(hot):
+                sel = rows_b[hb[:, h]]
+                prog[sel, k - 1 - filled[sel]] = h
+                filled[sel] += 1
+        idx[big] = prog
+    if empty_frac > 0:
+        idx[torch.rand(rows, k, generator=g) < empty_frac] = -1
+    # the slot order within a row carries no meaning; shuffle the short rows' slots
+    if bool(small.any()):
+        sr = torch.nonzero(small).flatten()
+        perm = torch.argsort(torch.rand(sr.numel(), k, generator=g), dim=1)
+        idx[sr] = torch.gather(idx[sr], 1, perm)
+    return idx.to(torch.int32).contiguous()

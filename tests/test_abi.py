@@ -76,3 +76,47 @@ def test_attention_workspace_does_not_grow_with_the_sequence():
     assert T.topk_attn_workspace_bytes(1, 12, 4096, 4096, 64, 256, 1024, 1) == 0
     # invalid arguments report 0
     assert T.topk_attn_workspace_bytes(1, 12, 4096, 4096, 64, 0, 1024, 1) == 0
+
+
+def _attn_bwd(lib, **kw):
+    a = dict(q=16, k=16, v=16, dout=16, idx=16, score=16, dq=16, dk=16, dv=16, B=1, H=1, Lq=8, Lk=8, d=64,
+             topk=4, dtype=1)
+    a.update(kw)
+    return lib.topk_attn_bwd(a["q"], a["k"], a["v"], a["dout"], a["idx"], a["score"], a["dq"], a["dk"], a["dv"],
+                             a["B"], a["H"], a["Lq"], a["Lk"], a["d"], a["topk"], a["dtype"], None)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(q=None), -1), (dict(dout=None), -1), (dict(idx=None), -1), (dict(dv=None), -1), (dict(B=0), -1),
+    (dict(topk=0), -1), (dict(topk=9), -1), (dict(dtype=5), -1), (dict(d=96), -2), (dict(dtype=0, d=48), -2),
+    (dict(topk=3000, Lk=4000), -2), (dict(dq=24), -2), (dict(idx=18), -2),
+    (dict(B=1 << 16, H=1 << 10, Lq=64, topk=4, Lk=8), -2),
+])
+def test_attention_backward_argument_errors(lib, kw, code):
+    assert _attn_bwd(lib, **kw) == code
+
+
+def test_ffn_backward_argument_errors(lib):
+    f = lib.topk_ffn_bwd
+    ok = [16] * 9
+    assert f(*([None] + ok[1:]), 4, 64, 128, 8, None) == -1
+    assert f(*ok, 4, 64, 128, 0, None) == -1
+    assert f(*ok, 4, 64, 128, 129, None) == -1
+    assert f(*ok, 4, 100, 128, 8, None) == -2
+    assert f(*ok, 4, 4096, 128, 8, None) == -2
+    assert f(*(ok[:6] + [24] + ok[7:]), 4, 64, 128, 8, None) == -2
+
+
+def test_backward_scratch_is_linear_in_the_cache():
+    # rank + entry per cached (row, slot): 20 bytes; count + offset per key: 8 bytes; nothing per (query, key)
+    def attn(L, k):
+        return T.topk_attn_bwd_workspace_bytes(1, 12, L, L, 64, k, 1)
+    for L in (8192, 65536):
+        ws = attn(L, 64)
+        entries, keys = 12 * L * 64, 12 * L
+        assert entries * 20 + keys * 8 <= ws <= entries * 20 + keys * 8 + 5 * 256 + 4 * (keys // 4096 + 1)
+    # doubling L doubles the growth (up to the 256-byte alignment of the parts): linear, no L^2 term
+    assert abs((attn(65536, 64) - attn(32768, 64)) - 2 * (attn(32768, 64) - attn(16384, 64))) <= 2048
+    f = T.topk_ffn_bwd_workspace_bytes
+    assert 4096 * 512 * 20 <= f(4096, 1024, 65536, 512) <= 4096 * 512 * 20 + 65536 * 8 + 4096
+    assert f(4096, 4096, 65536, 512) == 0 and attn(1024, 0) == 0
