@@ -13,6 +13,10 @@ is no collective on the data path ("replicas only", weak scaling).
 
 --impl reference times the CPU oracle (fp64, all host cores) on bounded
 samples of the same workload: the only other implementation there is.
+
+--pass bwd times the backward pass for the cached kept set instead (Sec. 2.2):
+the gradients of q, k, v (x, W1, W2) from dout and the forward pass's cache,
+and the training step forward-with-cache + backward.
 """
 from __future__ import annotations
 
@@ -47,6 +51,8 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU work budget of the oracle baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-clocks", action="store_true")
+    p.add_argument("--pass", dest="which", choices=["fwd", "bwd"], default="fwd",
+                   help="bwd: time the backward pass (Sec. 2.2) for the forward pass's cache instead")
     p.add_argument("--kernel-only", action="store_true",
                    help="time the device call only: no end-to-end leg, clocks or CPU baseline (profiling)")
     a = p.parse_args()
@@ -444,10 +450,149 @@ def run_ours(args):
         sys.exit("parity check of the timed output failed: " + line["parity"]["error"])
 
 
+# ------------------------------------------------------------------ backward pass
+BWD_METRIC = "top-k backward (cached kept set, Sec. 2.2) tokens/s"
+
+
+def bwd_bytes(w):
+    """Compulsory HBM bytes of one backward call: the inputs q, k, v, dout and the cache (idx, score)
+    read once, the fp32 gradients dq, dk, dv written once.  The gathered rows (k value and k key rows
+    per query row, k query and dout rows per kept entry) come mostly from L2 and are not counted."""
+    if w.kind == "ffn":
+        R, Lk, d, eb = w.N, w.d_ff, w.d_model, 2
+        return R * d * eb + 2 * Lk * d * eb + R * d * 4 + R * w.topk * 8 + (R * d + 2 * Lk * d) * 4
+    eb = 2 if w.dtype == "bf16" else 4
+    R, Lk = w.B * w.H * w.Lq, w.B * w.H * w.Lk
+    return (R + 2 * Lk + R) * w.d * eb + R * w.topk * 8 + (R + 2 * Lk) * w.d * 4
+
+
+def bwd_cpu_rate(w, host, dout, seconds):
+    """The oracle's backward pass on a bounded head slice (all host cores): tokens/s.  Its cache is a
+    random kept set (the backward pass is defined for any), not the CUDA forward pass's."""
+    import oracle
+    from paper_2106_06899_gb300 import workloads as W
+
+    cores = oracle.hardware_threads()
+    if w.kind == "ffn":
+        n = max(16, min(w.N, int(seconds * 40)))
+        idx = W.kept_sets(1, n, w.d_ff, w.topk, seed=7)
+        t0 = time.perf_counter()
+        oracle.ffn_bwd(host[0][:n], host[1], host[2], dout[:n].cpu(), idx.numpy())
+        t = time.perf_counter() - t0
+        return {"value": n / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                "sample": f"{n} of {w.N} tokens, random kept sets, fp64 oracle backward, {t:.1f} s"}
+    h = 1
+    q, k, v = (x[:, :h] for x in host)
+    idx = W.kept_sets(w.B * h, w.Lq, w.Lk, w.topk, seed=7)
+    t0 = time.perf_counter()
+    oracle.topk_attention_bwd(q.contiguous(), k.contiguous(), v.contiguous(), dout[:, :h].cpu().contiguous(),
+                              idx.numpy())
+    t = time.perf_counter() - t0
+    tokens = w.B * w.Lq * h / w.H
+    return {"value": tokens / t, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{h} of {w.H} heads (all rows), random kept sets, fp64 oracle backward, {t:.1f} s"}
+
+
+def run_backward(args):
+    """Times the backward pass for the CUDA forward pass's own cache (one forward call with index
+    output before timing), and the training step forward-with-cache + backward."""
+    import torch
+
+    from paper_2106_06899_gb300 import topk as T
+    from paper_2106_06899_gb300 import workloads as W
+
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    w = workload(args)
+    host = W.make_inputs(w)
+    dev = [t.cuda() for t in host]
+    if w.kind == "ffn":
+        dout = W.grad_output((w.N, w.d_model), dtype="f32", seed=w.seed + 1).cuda()
+        out, idx, score = T.ffn(dev[0], dev[1], dev[2], w.topk, return_indices=True)
+        grads = [torch.empty(t.shape, dtype=torch.float32, device="cuda") for t in dev]
+
+        def bwd():
+            T.topk_ffn_bwd(dev[0], dev[1], dev[2], dout, idx, score, *grads)
+
+        def fwd():
+            T.topk_ffn_fwd_indices(dev[0], dev[1], dev[2], out, w.topk, idx, score)
+    else:
+        dout = W.grad_output((w.B, w.H, w.Lq, w.d), dtype=w.dtype, seed=w.seed + 1).cuda()
+        out, idx, score = T.attention(dev[0], dev[1], dev[2], w.topk, w.chunk, w.causal, return_indices=True)
+        grads = [torch.empty(t.shape, dtype=torch.float32, device="cuda") for t in dev]
+
+        def bwd():
+            T.topk_attn_bwd(dev[0], dev[1], dev[2], dout, idx, score, *grads)
+
+        def fwd():
+            T.topk_attn_fwd_indices(dev[0], dev[1], dev[2], out, w.topk, w.chunk, w.causal, idx, score)
+    T.topk_check()
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def timed(fn):
+        for _ in range(args.warmup):
+            fn()
+        torch.cuda.synchronize()
+        tot = 0.0
+        for _ in range(args.steps):
+            flush.fill_(1.0)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            fn()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            tot += e0.elapsed_time(e1)
+        T.topk_check()
+        return tot / args.steps
+
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(0).uuid)
+    except Exception:
+        pass
+    sampler = ClockSampler(uuid)
+    if not args.no_clocks:
+        sampler.start()
+        time.sleep(0.3)
+    ms_bwd = timed(bwd)
+    launches = T.topk_last_launch_count()
+    ms_fwd = timed(fwd)
+
+    def train_step():
+        fwd()
+        bwd()
+
+    ms_train = timed(train_step)
+    clocks = None if args.no_clocks else sampler.stop()
+    pk = peaks()
+    nbytes = bwd_bytes(w)
+    achieved = nbytes / (ms_bwd / 1e3) / 1e9
+    line = {
+        "metric": BWD_METRIC, "value": w.tokens / (ms_bwd / 1e3), "unit": "tokens/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_bwd, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == "bf16" else "f32",
+        "data": "synthetic", "config": config_dict(w, "L2 flushed between steps (write of 2x L2 size)"),
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                     "frac": achieved / pk["hbm_gbs"], "traffic": None, "bytes_per_call": nbytes,
+                     "peak_source": f"{pk['source']} HBM copy bandwidth", "kernel": "backward kernels"},
+        "forward_with_cache_ms": ms_fwd,
+        "train_step_ms": ms_train,
+        "train_step_tokens_per_s": w.tokens / (ms_train / 1e3),
+        "gpu_launches": launches * args.steps,
+        "clocks": clocks,
+        "e2e": None,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = bwd_cpu_rate(w, host, dout, args.cpu_seconds)
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         run_reference(args)
+    elif args.which == "bwd":
+        run_backward(args)
     else:
         run_ours(args)
 
