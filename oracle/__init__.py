@@ -66,11 +66,15 @@ def _load():
             lib.oracle_vanilla.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i32, vp, i64, vp, i32]
             lib.oracle_eval_indices.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i64, vp, i64,
                                                 vp, vp, vp, vp, i32]
+            lib.oracle_topk_masked.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i64, i32, vp, vp,
+                                               i64, i64, vp, i64, vp, vp, vp, vp, i32]
+            lib.oracle_vanilla_masked.argtypes = [i32, i32, vp, vp, vp, i64, i64, i64, i64, i64, i32, vp, vp,
+                                                  i64, i64, vp, i64, vp, i32]
             lib.oracle_topk_bwd.argtypes = [i32, i32, vp, vp, vp, i32, vp, i64, i64, i64, i64, i64, i64, vp,
                                             vp, vp, vp, i32]
             lib.oracle_hardware_threads.argtypes = []
             for f in (lib.oracle_topk, lib.oracle_vanilla, lib.oracle_eval_indices, lib.oracle_topk_bwd,
-                      lib.oracle_hardware_threads):
+                      lib.oracle_topk_masked, lib.oracle_vanilla_masked, lib.oracle_hardware_threads):
                 f.restype = ctypes.c_int
             _lib = lib
     return _lib
@@ -121,8 +125,40 @@ def _common(q, k, v, act):
     return qa, ka, va, dt
 
 
-def topk_attention(q, k, v, topk: int, *, act: int = SOFTMAX, causal: bool = False, rows=None, threads: int = 0):
-    """Eq. 4 (act=SOFTMAX) or Eq. 3 (act=RELU) for q [B,H,Lq,d], k/v [B,H,Lk,d].
+def _masks(kv_len, mask, B, H, Lq, Lk):
+    """(kv_len int32 [B] or None, packed mask words or None, batch stride, head stride).
+
+    mask: boolean array of shape [B or 1, H or 1, Lq, Lk], True where the key is valid (Eq. 2's
+    B_ij = 0); a dimension of size 1 applies to every batch / head.  Packed here, independently of
+    the CUDA binding, as bit j % 32 of word j // 32 of each query row (little-endian bit order)."""
+    kl = None
+    if kv_len is not None:
+        kl = np.ascontiguousarray(np.asarray(kv_len, dtype=np.int32).reshape(B))
+    words = None
+    mbs = mhs = 0
+    if mask is not None:
+        m = np.asarray(mask, dtype=bool)
+        if m.ndim != 4 or m.shape[2:] != (Lq, Lk) or m.shape[0] not in (1, B) or m.shape[1] not in (1, H):
+            raise ValueError("mask must be [B or 1, H or 1, Lq, Lk]")
+        W = (Lk + 31) // 32
+        padded = np.zeros(m.shape[:3] + (W * 32,), bool)
+        padded[..., :Lk] = m
+        bits = padded.reshape(m.shape[:3] + (W, 32)).astype(np.uint64)
+        words = np.ascontiguousarray((bits << np.arange(32, dtype=np.uint64)).sum(axis=-1).astype(np.uint32))
+        mhs = Lq * W if m.shape[1] == H and H > 1 else 0
+        mbs = m.shape[1] * Lq * W if m.shape[0] == B and B > 1 else 0
+    return kl, words, mbs, mhs
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data
+
+
+def topk_attention(q, k, v, topk: int, *, act: int = SOFTMAX, causal: bool = False, rows=None, threads: int = 0,
+                   kv_len=None, mask=None):
+    """Eq. 4 (act=SOFTMAX) or Eq. 3 (act=RELU) for q [B,H,Lq,d], k/v [B,H,Lk,d], under the masks of
+    Eq. 2: causal (key j valid for query i iff j <= i + Lk - Lq; needs Lq <= Lk), kv_len ([B]: key j
+    valid iff j < kv_len[b]) and mask (boolean [B|1, H|1, Lq, Lk], True = valid).
 
     Returns dict(out [n,d] f64, idx [n,topk] i32 (-1 pad), score [n,topk] f64 (-inf pad),
     next_score [n] f64 (the (k+1)-th score, -inf if none)); n = len(rows) or B*H*Lq.
@@ -133,27 +169,31 @@ def topk_attention(q, k, v, topk: int, *, act: int = SOFTMAX, causal: bool = Fal
     if ka.shape != (B, H, Lk, d) or va.shape != (B, H, Lk, d):
         raise ValueError("shape mismatch")
     r, n, rp = _rows_arg(rows, B * H * Lq)
+    kl, words, mbs, mhs = _masks(kv_len, mask, B, H, Lq, Lk)
     out = np.zeros((n, d), np.float64)
     idx = np.zeros((n, topk), np.int32)
     score = np.zeros((n, topk), np.float64)
     nxt = np.zeros((n,), np.float64)
-    rc = _load().oracle_topk(act, dt, qa.ctypes.data, ka.ctypes.data, va.ctypes.data, B, H, Lq, Lk, d, topk,
-                             int(causal), rp, n, out.ctypes.data, idx.ctypes.data, score.ctypes.data,
-                             nxt.ctypes.data, threads)
+    rc = _load().oracle_topk_masked(act, dt, qa.ctypes.data, ka.ctypes.data, va.ctypes.data, B, H, Lq, Lk, d,
+                                    topk, int(causal), _ptr(kl), _ptr(words), mbs, mhs, rp, n, out.ctypes.data,
+                                    idx.ctypes.data, score.ctypes.data, nxt.ctypes.data, threads)
     if rc:
         raise RuntimeError(f"oracle_topk failed: {rc}")
     return {"out": out, "idx": idx, "score": score, "next_score": nxt}
 
 
-def vanilla(q, k, v, *, act: int = SOFTMAX, causal: bool = False, rows=None, threads: int = 0):
-    """Eq. 1 (softmax over all valid keys; causal mask of Eq. 2) -> out [n, d] f64."""
+def vanilla(q, k, v, *, act: int = SOFTMAX, causal: bool = False, rows=None, threads: int = 0, kv_len=None,
+            mask=None):
+    """Eq. 1 (softmax over all valid keys under the masks of Eq. 2, as in topk_attention) -> out [n, d] f64."""
     qa, ka, va, dt = _common(q, k, v, act)
     B, H, Lq, d = qa.shape
     Lk = ka.shape[2]
     r, n, rp = _rows_arg(rows, B * H * Lq)
+    kl, words, mbs, mhs = _masks(kv_len, mask, B, H, Lq, Lk)
     out = np.zeros((n, d), np.float64)
-    rc = _load().oracle_vanilla(act, dt, qa.ctypes.data, ka.ctypes.data, va.ctypes.data, B, H, Lq, Lk, d,
-                                int(causal), rp, n, out.ctypes.data, threads)
+    rc = _load().oracle_vanilla_masked(act, dt, qa.ctypes.data, ka.ctypes.data, va.ctypes.data, B, H, Lq, Lk, d,
+                                       int(causal), _ptr(kl), _ptr(words), mbs, mhs, rp, n, out.ctypes.data,
+                                       threads)
     if rc:
         raise RuntimeError(f"oracle_vanilla failed: {rc}")
     return out

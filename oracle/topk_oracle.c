@@ -11,7 +11,11 @@
  *
  *   Eq. 1  (dot-product attention, temperature folded into Q):
  *            s_ij = sum_t q_i[t] * k_j[t]
- *   Eq. 2  (masking): with the causal mask only keys j <= i are valid.
+ *   Eq. 2  (masking): a key j is valid for query i unless B_ij = -inf.  The
+ *          masks taken: causal (j <= i + Lk - Lq: the queries are the last
+ *          Lq positions of the sequence, as when decoding against a cache of
+ *          Lk keys), a key count per batch (j < kv_len[b]: key padding) and
+ *          an arbitrary bit mask (bit j of query row i: 1 = valid).
  *   Eq. 4  (top-k attention): keep the k largest s_ij of row i, apply the
  *            activation to those k entries only, and weight the value rows:
  *            out_i = sum_{j in topk(i)} act(s_i, topk(i))_j * v_j
@@ -22,8 +26,9 @@
  * Readings where the paper is silent (Sec. 2.2 gives none of these):
  *   - ties in s are broken toward the lower key index, i.e. the kept set is
  *     the first k entries of the total order (s descending, j ascending);
- *   - a causal row with fewer than k valid keys keeps all of them
- *     (k_eff = i + 1), and the softmax covers those only;
+ *   - a row with fewer than k valid keys keeps all of them (k_eff = the
+ *     number of valid keys), and the softmax covers those only; a row with
+ *     no valid key outputs zeros;
  *   - top-k runs on the signed scores; ReLU is applied after selection.
  *
  * Arithmetic: inputs are widened exactly to double (bf16 by a 16-bit
@@ -102,6 +107,10 @@ typedef struct {
   const void *q, *k, *v;
   int64_t H, Lq, Lk, d, topk;
   int causal, vanilla;
+  int64_t coff;            /* causal: key j is valid for query i iff j <= i + coff */
+  const int32_t* kv_len;   /* [B] valid keys per batch, or NULL */
+  const uint32_t* mask;    /* bit mask, or NULL: word (b*mbs + h*mhs + i*mw + j/32) */
+  int64_t mbs, mhs, mw;
   const int64_t* rows;
   int64_t nrows;
   const int32_t* eval_idx; /* index-evaluate mode when non-NULL */
@@ -110,6 +119,18 @@ typedef struct {
   int64_t begin, end;
   int status;
 } job;
+
+/* Eq. 2: is key j valid for query i of problem bh = b * H + h? */
+static int key_valid(const job* J, int64_t bh, int64_t i, int64_t j) {
+  const int64_t b = bh / J->H, h = bh % J->H;
+  if (J->causal && j > i + J->coff) return 0;
+  if (J->kv_len && j >= (int64_t)J->kv_len[b]) return 0;
+  if (J->mask) {
+    const uint32_t w = J->mask[b * J->mbs + h * J->mhs + i * J->mw + (j >> 5)];
+    if (!((w >> (j & 31)) & 1u)) return 0;
+  }
+  return 1;
+}
 
 static double dot_row(const job* J, int64_t krow, const double* qbuf) {
   double acc = 0.0;
@@ -132,7 +153,6 @@ static void* run_rows(void* arg) {
     const int64_t row = J->rows ? J->rows[r] : r;
     const int64_t bh = row / J->Lq, i = row % J->Lq;
     for (int64_t t = 0; t < d; ++t) qbuf[t] = widen(J->q, (size_t)(row * d + t), J->dtype);
-    const int64_t nvalid = J->causal ? (i + 1 < J->Lk ? i + 1 : J->Lk) : J->Lk;
     int64_t nsel = 0;
     double next = -INFINITY;
 
@@ -151,7 +171,8 @@ static void* run_rows(void* arg) {
       }
     } else if (J->vanilla) {
       /* Eq. 1 / Eq. 2: every valid key is kept. */
-      for (int64_t j = 0; j < nvalid; ++j) {
+      for (int64_t j = 0; j < J->Lk; ++j) {
+        if (!key_valid(J, bh, i, j)) continue;
         sel[nsel].j = (int32_t)j;
         sel[nsel].s = dot_row(J, bh * J->Lk + j, qbuf);
         nsel++;
@@ -159,7 +180,8 @@ static void* run_rows(void* arg) {
     } else {
       /* Eq. 4: bounded heap of the K+1 highest-ranked entries. */
       int64_t cap = K + 1, n = 0;
-      for (int64_t j = 0; j < nvalid; ++j) {
+      for (int64_t j = 0; j < J->Lk; ++j) {
+        if (!key_valid(J, bh, i, j)) continue;
         entry e;
         e.j = (int32_t)j;
         e.s = dot_row(J, bh * J->Lk + j, qbuf);
@@ -249,15 +271,33 @@ static int run(job proto, int nthreads) {
   return status;
 }
 
+/* Mask arguments shared by the entry points (Eq. 2): causal (requires
+ * Lq <= Lk; key j is valid for query i iff j <= i + Lk - Lq), kv_len
+ * ([B] int32 or NULL; key j valid iff j < kv_len[b]) and mask (uint32 bit
+ * words or NULL; bit j % 32 of word b*mbs + h*mhs + i*ceil(Lk/32) + j/32;
+ * 1 = valid).  All three apply together. */
+static int set_masks(job* J, int64_t Lq, int64_t Lk, int causal, const int32_t* kv_len, const uint32_t* mask,
+                     int64_t mbs, int64_t mhs) {
+  if (causal && Lq > Lk) return -2;
+  J->causal = causal;
+  J->coff = Lk - Lq;
+  J->kv_len = kv_len;
+  J->mask = mask;
+  J->mbs = mbs;
+  J->mhs = mhs;
+  J->mw = (Lk + 31) / 32;
+  return 0;
+}
+
 /* Top-k attention (Eq. 4) or, with act = ACT_RELU and B = H = 1, the
- * top-k feed-forward layer (Eq. 3).  Rows are flattened (b, h, i) indices
- * into [B*H*Lq]; rows == NULL means all of them in order.
- * Outputs per listed row: out [d], idx [topk] (-1 padded), score [topk]
- * (-inf padded), next_score = the (k+1)-th score or -inf. */
-int oracle_topk(int act, int dtype, const void* q, const void* k, const void* v, int64_t B, int64_t H,
-                int64_t Lq, int64_t Lk, int64_t d, int64_t topk, int causal, const int64_t* rows,
-                int64_t nrows, double* out, int32_t* idx, double* score, double* next_score,
-                int nthreads) {
+ * top-k feed-forward layer (Eq. 3), under the masks above.  Rows are
+ * flattened (b, h, i) indices into [B*H*Lq]; rows == NULL means all of them
+ * in order.  Outputs per listed row: out [d], idx [topk] (-1 padded), score
+ * [topk] (-inf padded), next_score = the (k+1)-th score or -inf. */
+int oracle_topk_masked(int act, int dtype, const void* q, const void* k, const void* v, int64_t B, int64_t H,
+                       int64_t Lq, int64_t Lk, int64_t d, int64_t topk, int causal, const int32_t* kv_len,
+                       const uint32_t* mask, int64_t mbs, int64_t mhs, const int64_t* rows, int64_t nrows,
+                       double* out, int32_t* idx, double* score, double* next_score, int nthreads) {
   job J;
   memset(&J, 0, sizeof J);
   J.act = act;
@@ -270,22 +310,30 @@ int oracle_topk(int act, int dtype, const void* q, const void* k, const void* v,
   J.Lk = Lk;
   J.d = d;
   J.topk = topk;
-  J.causal = causal;
   J.rows = rows;
   J.nrows = rows ? nrows : B * H * Lq;
   J.out = out;
   J.idx = idx;
   J.score = score;
   J.next_score = next_score;
-  if (causal && Lq != Lk) return -2;
+  if (set_masks(&J, Lq, Lk, causal, kv_len, mask, mbs, mhs)) return -2;
   return run(J, nthreads);
 }
 
-/* Plain attention over every valid key (Eq. 1, with the causal mask of
- * Eq. 2 when causal != 0).  Same row convention as oracle_topk. */
-int oracle_vanilla(int act, int dtype, const void* q, const void* k, const void* v, int64_t B, int64_t H,
-                   int64_t Lq, int64_t Lk, int64_t d, int causal, const int64_t* rows, int64_t nrows,
-                   double* out, int nthreads) {
+int oracle_topk(int act, int dtype, const void* q, const void* k, const void* v, int64_t B, int64_t H,
+                int64_t Lq, int64_t Lk, int64_t d, int64_t topk, int causal, const int64_t* rows,
+                int64_t nrows, double* out, int32_t* idx, double* score, double* next_score,
+                int nthreads) {
+  return oracle_topk_masked(act, dtype, q, k, v, B, H, Lq, Lk, d, topk, causal, NULL, NULL, 0, 0, rows, nrows,
+                            out, idx, score, next_score, nthreads);
+}
+
+/* Plain attention over every valid key (Eq. 1 under the masks of Eq. 2).
+ * Same row convention as oracle_topk. */
+int oracle_vanilla_masked(int act, int dtype, const void* q, const void* k, const void* v, int64_t B,
+                          int64_t H, int64_t Lq, int64_t Lk, int64_t d, int causal, const int32_t* kv_len,
+                          const uint32_t* mask, int64_t mbs, int64_t mhs, const int64_t* rows, int64_t nrows,
+                          double* out, int nthreads) {
   job J;
   memset(&J, 0, sizeof J);
   J.act = act;
@@ -298,13 +346,19 @@ int oracle_vanilla(int act, int dtype, const void* q, const void* k, const void*
   J.Lk = Lk;
   J.d = d;
   J.topk = Lk;
-  J.causal = causal;
   J.vanilla = 1;
   J.rows = rows;
   J.nrows = rows ? nrows : B * H * Lq;
   J.out = out;
-  if (causal && Lq != Lk) return -2;
+  if (set_masks(&J, Lq, Lk, causal, kv_len, mask, mbs, mhs)) return -2;
   return run(J, nthreads);
+}
+
+int oracle_vanilla(int act, int dtype, const void* q, const void* k, const void* v, int64_t B, int64_t H,
+                   int64_t Lq, int64_t Lk, int64_t d, int causal, const int64_t* rows, int64_t nrows,
+                   double* out, int nthreads) {
+  return oracle_vanilla_masked(act, dtype, q, k, v, B, H, Lq, Lk, d, causal, NULL, NULL, 0, 0, rows, nrows, out,
+                               nthreads);
 }
 
 /* Index-evaluate: the kept set of each listed row is given in idx
