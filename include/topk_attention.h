@@ -7,8 +7,12 @@
  *   topk_attn_fwd  -- Eq. 4 (Sec. 2.2):  out = softmax(top-k(Q K^T)) V, row by
  *                     row, the softmax taken over the k kept entries only.
  *                     The temperature of Eq. 1 is folded into Q by the caller
- *                     (footnote to Eq. 1).  Optional causal mask, Eq. 2: key j
- *                     is valid for query i iff j <= i.
+ *                     (footnote to Eq. 1).  Optional causal mask, Eq. 2: the
+ *                     queries are the last Lq of the Lk positions (Lq <= Lk;
+ *                     Lq < Lk is decoding against a key/value cache), and key
+ *                     j is valid for query i iff j <= i + Lk - Lq.
+ *   topk_attn_fwd_masked -- the same under Eq. 2's general mask B in {0, -inf}:
+ *                     per-batch key counts and an arbitrary bit mask as well.
  *   topk_ffn_fwd   -- Eq. 3 with top-k (Sec. 2.1 "Feed-forward as attention"):
  *                     out = sum over the k largest s_j = x . W1_j of
  *                     ReLU(s_j) * W2_j.  Keys and values are the ROWS of W1
@@ -23,8 +27,9 @@
  * in device memory.
  *
  * Selection rule: each row keeps the first k entries of the total order
- * (score descending, key index ascending), i.e. ties go to the lower key
- * index.  A causal row i with fewer than k valid keys keeps all i+1 of them.
+ * (score descending, key index ascending) among its valid keys, i.e. ties go
+ * to the lower key index.  A row with fewer than k valid keys keeps all of
+ * them; a row with none outputs zeros (its indices are all -1).
  *
  * Conventions shared by every call
  *   - Tensor pointers are DEVICE pointers (except the *_host entry points),
@@ -67,7 +72,7 @@ typedef enum { TOPK_F32 = 0, TOPK_BF16 = 1 } topk_dtype;
 enum {
   TOPK_OK = 0,
   TOPK_ERR_INVALID_ARG = -1, /* null pointer, non-positive size, topk < 1 or > keys, chunk < 1,
-                                causal with Lq != Lk, unknown dtype */
+                                causal with Lq > Lk, negative mask stride, unknown dtype */
   TOPK_ERR_UNSUPPORTED = -2, /* valid but not implemented: head size, topk above the
                                 kernel's limit, pointer not 16-byte aligned */
   TOPK_ERR_CUDA = -3,        /* a CUDA runtime/driver call or a launch failed */
@@ -86,7 +91,7 @@ enum {
  * Top-k attention forward, Eq. 4 (Sec. 2.2), optionally causal (Eq. 2).
  *   q, k, v, out : device pointers, layouts above, element type `dtype`.
  *   B, H         : batch and heads; every (b, h) is an independent problem.
- *   Lq, Lk       : query and key counts (causal requires Lq == Lk).
+ *   Lq, Lk       : query and key counts (causal requires Lq <= Lk).
  *   d            : head size.  TOPK_BF16: 64 or 128.  TOPK_F32: 16, 32, 64, 128.
  *   topk         : 1 <= topk <= Lk; the supported maximum is 512.
  *   chunk        : query-chunk size (Sec. 2.2), >= 1; a scheduling hint only.
@@ -110,6 +115,31 @@ int topk_attn_fwd(const void* q, const void* k, const void* v, void* out, int B,
 int topk_attn_fwd_indices(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq,
                           int Lk, int d, int topk, int chunk, int causal, int dtype, int32_t* idx,
                           float* score, void* stream);
+
+/*
+ * Top-k attention under the general mask of Eq. 2 (Sec. 2.1): B_ij = -inf
+ * removes key j from query i's candidates before the top-k.  Three masks
+ * combine (a key must pass all of them):
+ *   causal  : 0 or 1, as in topk_attn_fwd (key j valid iff j <= i + Lk - Lq).
+ *   kv_len  : NULL, or [B] int32 device pointer: key j is valid for every query
+ *             of batch b iff j < kv_len[b] (key padding; values are clamped to
+ *             [0, Lk]).
+ *   mask    : NULL, or a uint32 device bit array: key j is valid for query i of
+ *             (b, h) iff bit (j % 32) of word
+ *               b * mask_batch_stride + h * mask_head_stride + i * W + j / 32,
+ *             W = ceil(Lk / 32), is 1.  A stride of 0 shares the mask across
+ *             batches or heads.  4-byte aligned.
+ * A row with fewer than k valid keys keeps all of them; a row with none writes
+ * zeros.  Other arguments as topk_attn_fwd_indices (idx/score may be NULL).
+ * With a bit mask the scores run on the CUDA cores (fp32 FMA of the exact
+ * bf16/fp32 inputs); causal and kv_len alone keep the tensor-core kernel.
+ * Errors: as topk_attn_fwd; a negative stride is TOPK_ERR_INVALID_ARG, a
+ * misaligned mask or kv_len TOPK_ERR_UNSUPPORTED.
+ */
+int topk_attn_fwd_masked(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk,
+                         int d, int topk, int chunk, int causal, const int32_t* kv_len, const uint32_t* mask,
+                         long long mask_batch_stride, long long mask_head_stride, int dtype, int32_t* idx,
+                         float* score, void* stream);
 
 /*
  * Top-k feed-forward layer, Eq. 3 with the top-k of Eq. 4 and ReLU as the

@@ -40,14 +40,14 @@ def _delta(q_rows: np.ndarray, k_all: torch.Tensor, d: int) -> np.ndarray:
 
 
 def check_rows(*, q, k, v, rows, gpu_out, gpu_idx, gpu_score, topk, dtype, act=SOFTMAX, causal=False,
-               tol=None, ref=None):
+               tol=None, ref=None, kv_len=None, mask=None):
     """q/k/v: CPU tensors [B,H,L,d]; rows: flattened row ids; gpu_*: CPU arrays for those rows;
-    ref: the oracle's topk_attention result for those rows, if already computed.
-    Returns a dict of statistics; raises AssertionError on a violation."""
+    ref: the oracle's topk_attention result for those rows, if already computed; kv_len / mask: Eq. 2's
+    masks as the oracle takes them.  Returns a dict of statistics; raises AssertionError on a violation."""
     tol = TOL[dtype] if tol is None else tol
     rows = np.asarray(rows, dtype=np.int64)
     if ref is None:
-        ref = topk_attention(q, k, v, topk, act=act, causal=causal, rows=rows)
+        ref = topk_attention(q, k, v, topk, act=act, causal=causal, rows=rows, kv_len=kv_len, mask=mask)
     gi = np.asarray(gpu_idx, dtype=np.int32).reshape(len(rows), topk)
     gs = np.asarray(gpu_score, dtype=np.float64).reshape(len(rows), topk)
     go = np.asarray(gpu_out, dtype=np.float64).reshape(len(rows), -1)
@@ -64,7 +64,17 @@ def check_rows(*, q, k, v, rows, gpu_out, gpu_idx, gpu_score, topk, dtype, act=S
         assert len(set(gi[r, :n].tolist())) == n, "duplicate index"
     if causal:
         i = (rows % Lq)[:, None]
-        assert np.all((gi == -1) | (gi <= i)), "causal mask violated"
+        assert np.all((gi == -1) | (gi <= i + Lk - Lq)), "causal mask violated"
+    if kv_len is not None:
+        n_b = np.asarray(kv_len, dtype=np.int64)[rows // (H * Lq)][:, None]
+        assert np.all((gi == -1) | (gi < n_b)), "key count violated"
+    if mask is not None:
+        m = np.asarray(mask, dtype=bool)
+        for r in range(len(rows)):
+            b, h, i_r = rows[r] // (H * Lq), (rows[r] // Lq) % H, rows[r] % Lq
+            mr = m[b if m.shape[0] > 1 else 0, h if m.shape[1] > 1 else 0, i_r]
+            picks = gi[r][gi[r] >= 0]
+            assert np.all(mr[picks]), "bit mask violated"
 
     # order of the GPU list: its own scores non-increasing, equal scores by ascending index
     for r in range(len(rows)):

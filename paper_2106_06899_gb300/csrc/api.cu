@@ -112,7 +112,10 @@ int validate_attn(const AttnArgs& a) {
   if (a.B <= 0 || a.H <= 0 || a.Lq <= 0 || a.Lk <= 0 || a.d <= 0) return TOPK_ERR_INVALID_ARG;
   if (a.topk < 1 || a.topk > a.Lk || a.chunk < 1) return TOPK_ERR_INVALID_ARG;
   if (a.causal != 0 && a.causal != 1) return TOPK_ERR_INVALID_ARG;
-  if (a.causal && a.Lq != a.Lk) return TOPK_ERR_INVALID_ARG;
+  if (a.causal && a.Lq > a.Lk) return TOPK_ERR_INVALID_ARG;
+  if (a.mask_bs < 0 || a.mask_hs < 0) return TOPK_ERR_INVALID_ARG;
+  if (reinterpret_cast<uintptr_t>(a.mask) & 3u) return TOPK_ERR_UNSUPPORTED;
+  if (a.kv_len && (reinterpret_cast<uintptr_t>(a.kv_len) & 3u)) return TOPK_ERR_UNSUPPORTED;
   if (a.dtype != TOPK_F32 && a.dtype != TOPK_BF16) return TOPK_ERR_INVALID_ARG;
   const long long BH = static_cast<long long>(a.B) * a.H;
   if (BH > (1 << 30) || static_cast<long long>(a.Lq) * BH > (1ll << 40)) return TOPK_ERR_UNSUPPORTED;
@@ -275,6 +278,19 @@ int topk_attn_fwd_indices(const void* q, const void* k, const void* v, void* out
                           void* stream) {
   if ((idx && !aligned16(idx)) || (score && !aligned16(score))) return TOPK_ERR_UNSUPPORTED;
   AttnArgs a{q, k, v, out, B, H, Lq, Lk, d, topk, chunk, causal, dtype, idx, score};
+  return run_attn(a, static_cast<cudaStream_t>(stream));
+}
+
+int topk_attn_fwd_masked(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk,
+                         int d, int topk, int chunk, int causal, const int32_t* kv_len, const uint32_t* mask,
+                         long long mask_batch_stride, long long mask_head_stride, int dtype, int32_t* idx,
+                         float* score, void* stream) {
+  if ((idx && !aligned16(idx)) || (score && !aligned16(score))) return TOPK_ERR_UNSUPPORTED;
+  AttnArgs a{q, k, v, out, B, H, Lq, Lk, d, topk, chunk, causal, dtype, idx, score};
+  a.kv_len = kv_len;
+  a.mask = mask;
+  a.mask_bs = mask_batch_stride;
+  a.mask_hs = mask_head_stride;
   return run_attn(a, static_cast<cudaStream_t>(stream));
 }
 

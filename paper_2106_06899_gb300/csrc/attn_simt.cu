@@ -6,7 +6,7 @@
 // owns one query row for the whole pass: the row's query vector sits in
 // registers, key tiles of 32 rows are staged in shared memory and read by
 // broadcast, and the row's top-k is kept in a shared-memory heap
-// (select.cuh).  After the last key tile the softmax over the k kept scores
+// (select.cuh).  It also serves the arbitrary bit masks of Eq. 2.  After the last key tile the softmax over the k kept scores
 // and the weighted sum of their value rows are written out.  No score matrix
 // is stored anywhere.
 #include "kernels.h"
@@ -33,8 +33,11 @@ __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 x) {
 template <typename T, int D, int ROWS>
 __global__ void __launch_bounds__(ROWS) attn_simt_kernel(const T* __restrict__ q, const T* __restrict__ k,
                                                          const T* __restrict__ v, T* __restrict__ out, int BH,
-                                                         int Lq, int Lk, int topk, int causal,
-                                                         int32_t* __restrict__ idx, float* __restrict__ score) {
+                                                         int H, int Lq, int Lk, int topk, int causal,
+                                                         const int32_t* __restrict__ kv_len,
+                                                         const uint32_t* __restrict__ mask, long long mask_bs,
+                                                         long long mask_hs, int32_t* __restrict__ idx,
+                                                         float* __restrict__ score) {
   extern __shared__ __align__(16) uint8_t smem_raw[];
   float* ks = reinterpret_cast<float*>(smem_raw);                       // [KT][D]
   uint8_t* sel_mem = smem_raw + KT * D * sizeof(float);  // heap [topk][ROWS], records [GROUPS][ROWS]
@@ -58,10 +61,19 @@ __global__ void __launch_bounds__(ROWS) attn_simt_kernel(const T* __restrict__ q
   RowHeap<ROWS> heap;
   heap.init(sel_mem, tid, topk, GROUPS);
 
-  const int kend = causal ? min(Lk, (qt + 1) * ROWS) : Lk;
-  const uint32_t lim = static_cast<uint32_t>(causal ? min(i + 1, Lk) : Lk);
-  const int cta_lim_min = causal ? min(qt * ROWS + 1, Lk) : Lk;  // smallest limit in this CTA
+  // Eq. 2's masks.  Causal: the queries are the last Lq positions, key j is
+  // valid for query i iff j <= i + Lk - Lq.  kv_len: the batch's key count.
+  // Both give each row a valid key prefix [0, lim); the bit mask (1 = valid)
+  // then removes keys anywhere in it.
+  const int coff = Lk - Lq;
+  const int kv_end = kv_len ? min(max(__ldg(kv_len + bh / H), 0), Lk) : Lk;
+  const int kend = min(kv_end, causal ? (qt + 1) * ROWS + coff : Lk);
+  const uint32_t lim = static_cast<uint32_t>(min(kv_end, causal ? min(i + 1 + coff, Lk) : Lk));
+  const int cta_lim_min = min(kv_end, causal ? min(qt * ROWS + 1 + coff, Lk) : Lk);  // smallest limit here
   const T* kb = k + static_cast<size_t>(bh) * Lk * D;
+  const uint32_t* mrow = nullptr;
+  if (mask && row_ok)
+    mrow = mask + (bh / H) * mask_bs + (bh % H) * mask_hs + static_cast<long long>(i) * ((Lk + 31) / 32);
 
   for (int j0 = 0; j0 < kend; j0 += KT) {
     __syncthreads();
@@ -85,6 +97,13 @@ __global__ void __launch_bounds__(ROWS) attn_simt_kernel(const T* __restrict__ q
       }
     }
     if (j0 + KT > cta_lim_min) mask_scores(s, static_cast<uint32_t>(j0), lim);
+    if (mask) {
+      static_assert(KT == 32, "one mask word per key tile");
+      const uint32_t bits = mrow ? __ldg(mrow + j0 / 32) : 0u;
+#pragma unroll
+      for (int e = 0; e < KT; ++e)
+        if (!((bits >> e) & 1u)) s[e] = -INFINITY;
+    }
     heap.offer(s, static_cast<uint32_t>(j0));
   }
 
@@ -110,7 +129,7 @@ int launch_simt(const AttnArgs& a, cudaStream_t st) {
   const long long grid = static_cast<long long>(BH) * n_qt;
   kern<<<static_cast<unsigned>(grid), ROWS, smem, st>>>(
       static_cast<const T*>(a.q), static_cast<const T*>(a.k), static_cast<const T*>(a.v), static_cast<T*>(a.out),
-      BH, a.Lq, a.Lk, a.topk, a.causal, a.idx, a.score);
+      BH, a.H, a.Lq, a.Lk, a.topk, a.causal, a.kv_len, a.mask, a.mask_bs, a.mask_hs, a.idx, a.score);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 

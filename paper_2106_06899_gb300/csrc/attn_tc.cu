@@ -184,8 +184,9 @@ __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, const
 template <int D, int FK, bool SPLIT>
 __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmk,
-                   const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ out, int BH, int Lq, int Lk,
-                   int topk, int rec_cap, int causal, int n_units, int32_t* __restrict__ idx,
+                   const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ out, int BH, int H, int Lq,
+                   int Lk, int topk, int rec_cap, int causal, const int32_t* __restrict__ kv_len, int n_units,
+                   int32_t* __restrict__ idx,
                    float* __restrict__ score, uint64_t* __restrict__ park, int* __restrict__ park_n, DevCtl ctl) {
   using L = Layout<D, FK, SPLIT>;
   using Sel = typename L::Sel;
@@ -252,9 +253,22 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
       qt = u % n_qt;
     }
   };
-  auto key_tiles = [&](int qt) {
-    const int kend = causal ? min(Lk, (qt + 1) * BM) : Lk;
+  // Eq. 2's masks as a valid key prefix per row: causal (queries are the
+  // last Lq positions: key j is valid for query i iff j <= i + Lk - Lq) and
+  // the batch's key count.  A unit streams at least one key tile, all of it
+  // masked if its rows have no key, so that every pipeline stage runs.
+  const int coff = Lk - Lq;
+  auto kv_end = [&](int bh) { return kv_len ? min(max(__ldg(kv_len + bh / H), 0), Lk) : Lk; };
+  auto key_tiles = [&](int bh, int qt) {
+    int kend = min(kv_end(bh), causal ? (qt + 1) * BM + coff : Lk);
+    kend = max(kend, 1);
     return (kend + N - 1) / N;
+  };
+  auto row_limit = [&](int bh, int i) {  // keys j < limit are valid for query i
+    return static_cast<uint32_t>(min(kv_end(bh), causal ? min(i + 1 + coff, Lk) : Lk));
+  };
+  auto tile_limit_min = [&](int bh, int qt) {  // the smallest row limit of query tile qt
+    return min(kv_end(bh), causal ? min(qt * BM + 1 + coff, Lk) : Lk);
   };
 
   if (warp == 0) {
@@ -277,7 +291,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         for (int r = 0; r < R; ++r) tma_load_3d(q_s + r * BM * 128, &tmq, q_full, r * 64, qt * BM, bh);
       }
       ++q_issued;
-      const int nk = key_tiles(qt);
+      const int nk = key_tiles(bh, qt);
       for (int kt = 0; kt < nk; ++kt) {
         const int s = it % S;
         const uint32_t ph = (it / S) & 1u;
@@ -320,7 +334,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         break;
       }
       tc_fence_after();
-      const int nk = key_tiles(qt);
+      const int nk = key_tiles(bh, qt);
       for (int kt = 0; kt < nk; ++kt, ++it, ++acc_it) {
         const int s = it % S;
         if (!warp_wait(&full_k[s], (it / S) & 1u, ctl, abort_flag)) {
@@ -373,9 +387,9 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
       decode(u, bh, qt);
       f.begin_unit();
       const int i_row = qt * BM + row;
-      const int nk = key_tiles(qt);
-      const uint32_t lim = static_cast<uint32_t>(causal ? min(i_row + 1, Lk) : Lk);
-      const int lim_min = causal ? min(qt * BM + 1, Lk) : Lk;
+      const int nk = key_tiles(bh, qt);
+      const uint32_t lim = row_limit(bh, i_row);
+      const int lim_min = tile_limit_min(bh, qt);
       for (int kt = 0; ok && kt < nk; ++kt, ++acc_it) {
         const int b = acc_it % NACC;
         if (!warp_wait(&acc_full[b], (acc_it / NACC) & 1u, ctl, abort_flag)) {
@@ -490,7 +504,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         const int i_row = qt * BM + q * 32 + lane;
         const size_t slot = (static_cast<size_t>(blockIdx.x) * 4 + q) * 2 + (s & 1u);
         const int n = __ldcg(park_n + slot * 32 + lane);
-        if (i_row < Lq && n > 0) {
+        if (i_row < Lq) {  // a row without a valid key (n = 0) gets zeros
           const size_t orow = static_cast<size_t>(bh) * Lq + i_row;
           const ParkedKeys kept{park + slot * topk * 32 + lane, n};
           softmax_gather_store<__nv_bfloat16, D>(kept, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
@@ -512,9 +526,9 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
       decode(u, bh, qt);
       const int i_row = qt * BM + row;
       heap.init(sel_mem, row, topk, rec_cap);
-      const int nk = key_tiles(qt);
-      const uint32_t lim = static_cast<uint32_t>(causal ? min(i_row + 1, Lk) : Lk);
-      const int lim_min = causal ? min(qt * BM + 1, Lk) : Lk;
+      const int nk = key_tiles(bh, qt);
+      const uint32_t lim = row_limit(bh, i_row);
+      const int lim_min = tile_limit_min(bh, qt);
       for (int kt = 0; kt < nk; ++kt, ++acc_it) {
         const int b = acc_it % NACC;
         if (!warp_wait(&acc_full[b], (acc_it / NACC) & 1u, ctl, abort_flag)) {
@@ -588,8 +602,9 @@ int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t 
     park_n = reinterpret_cast<int*>(park + static_cast<size_t>(grid) * park_keys_per_cta(a.topk));
   }
   kern<<<grid, kThreads<SPLIT>, smem, st>>>(tmq, tmk, static_cast<const __nv_bfloat16*>(a.v),
-                                            static_cast<__nv_bfloat16*>(a.out), BH, a.Lq, a.Lk, a.topk,
-                                            L::cap(a.topk), a.causal, n_units, a.idx, a.score, park, park_n, ctl);
+                                            static_cast<__nv_bfloat16*>(a.out), BH, a.H, a.Lq, a.Lk, a.topk,
+                                            L::cap(a.topk), a.causal, a.kv_len, n_units, a.idx, a.score, park,
+                                            park_n, ctl);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
@@ -626,7 +641,7 @@ int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st
 }  // namespace
 
 bool attn_tc_supports(const AttnArgs& a) {
-  if (a.dtype != 1 || a.topk > kTcMaxK) return false;
+  if (a.dtype != 1 || a.topk > kTcMaxK || a.mask) return false;  // bit masks run on the SIMT kernel
   if (a.d == 64) return Layout<64, 0, false>::fits(a.topk);
   if (a.d == 128) return Layout<128, 0, false>::fits(a.topk);
   return false;

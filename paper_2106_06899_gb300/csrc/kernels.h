@@ -28,6 +28,12 @@ struct AttnArgs {
   // device scratch of the tcgen05 split kernel (attn_tc_workspace_bytes)
   void* workspace = nullptr;
   size_t workspace_bytes = 0;
+  // Eq. 2's masks besides causal: the key count of each batch ([B] int32,
+  // key j valid iff j < kv_len[b]) and a bit mask (bit j % 32 of word
+  // b * mask_bs + h * mask_hs + i * ceil(Lk / 32) + j / 32, 1 = valid)
+  const int32_t* kv_len = nullptr;
+  const uint32_t* mask = nullptr;
+  long long mask_bs = 0, mask_hs = 0;
 };
 
 struct FfnArgs {

@@ -49,6 +49,8 @@ def lib() -> ctypes.CDLL:
             L.topk_attn_workspace_bytes.restype = sz
             L.topk_ffn_workspace_bytes.argtypes = [i32] * 4
             L.topk_ffn_workspace_bytes.restype = sz
+            L.topk_attn_fwd_masked.argtypes = [vp, vp, vp, vp] + [i32] * 8 + [vp, vp, ctypes.c_longlong,
+                                                                            ctypes.c_longlong, i32, vp, vp, vp]
             L.topk_attn_bwd.argtypes = [vp] * 9 + [i32] * 7 + [vp]
             L.topk_ffn_bwd.argtypes = [vp] * 9 + [i32] * 4 + [vp]
             L.topk_attn_bwd_workspace_bytes.argtypes = [i32] * 7
@@ -68,7 +70,7 @@ def lib() -> ctypes.CDLL:
                       "topk_attn_fwd_host", "topk_ffn_fwd_host", "topk_ffn_fwd_noalloc", "topk_check",
                       "topk_last_launch_count",
                       "topk_debug_skip_arrive", "topk_pool_usage", "topk_pool_trim", "topk_attn_bwd",
-                      "topk_ffn_bwd"):
+                      "topk_ffn_bwd", "topk_attn_fwd_masked"):
                 getattr(L, f).restype = i32
             _lib = L
     return _lib
@@ -134,6 +136,47 @@ def topk_attn_fwd_indices(q, k, v, out, topk: int, chunk: int = 1024, causal: bo
     rc = lib().topk_attn_fwd_indices(_ptr(q), _ptr(k), _ptr(v), _ptr(out), B, H, Lq, Lk, d, int(topk), int(chunk),
                                      int(bool(causal)), _dtype_code(q), _ptr(idx), _ptr(score), _stream(stream))
     _check(rc, "topk_attn_fwd_indices")
+
+
+def pack_mask(mask: torch.Tensor):
+    """A boolean mask [B or 1, H or 1, Lq, Lk] (True = the key takes part, Eq. 2's B_ij = 0) in the
+    C ABI's layout: bit j % 32 of int32 word j // 32 of each query row, on mask's device.
+
+    Returns (words [B|1, H|1, Lq, ceil(Lk/32)] int32, batch stride, head stride) in words; a stride is
+    0 where the mask has one entry for all batches or heads."""
+    if mask.dim() != 4 or mask.dtype != torch.bool:
+        raise ValueError("mask must be a 4-D bool tensor [B or 1, H or 1, Lq, Lk]")
+    mb, mh, Lq, Lk = mask.shape
+    W = (Lk + 31) // 32
+    padded = torch.zeros(mb, mh, Lq, W * 32, dtype=torch.int64, device=mask.device)
+    padded[..., :Lk] = mask.to(torch.int64)
+    shifts = torch.arange(32, dtype=torch.int64, device=mask.device)
+    words = (padded.view(mb, mh, Lq, W, 32) << shifts).sum(dim=-1)
+    words = torch.where(words >= 2**31, words - 2**32, words).to(torch.int32).contiguous()
+    hs = Lq * W if mh > 1 else 0
+    bs = mh * Lq * W if mb > 1 else 0
+    return words, bs, hs
+
+
+def topk_attn_fwd_masked(q, k, v, out, topk: int, chunk: int = 1024, causal: bool = False, kv_len=None,
+                         mask_words=None, mask_batch_stride: int = 0, mask_head_stride: int = 0, idx=None,
+                         score=None, stream=None) -> None:
+    """Eq. 4 under Eq. 2's masks: causal (queries are the last Lq positions), kv_len [B] int32 (keys per
+    batch) and a packed bit mask (see pack_mask); idx/score as topk_attn_fwd_indices, or None."""
+    B, H, Lq, Lk, d = _attn_dims(q, k, v, out)
+    if kv_len is not None and (kv_len.dtype != torch.int32 or tuple(kv_len.shape) != (B,)):
+        raise ValueError("kv_len must be a [B] int32 tensor")
+    if mask_words is not None:
+        W = (Lk + 31) // 32
+        if mask_words.dtype != torch.int32 or not mask_words.is_contiguous() or mask_words.shape[-2:] != (Lq, W):
+            raise ValueError("mask_words must be a contiguous int32 [..., Lq, ceil(Lk/32)] tensor (pack_mask)")
+    for name, t, dt in (("idx", idx, torch.int32), ("score", score, torch.float32)):
+        if t is not None and (t.dtype != dt or tuple(t.shape) != (B, H, Lq, topk) or not t.is_contiguous()):
+            raise ValueError(f"{name} must be a contiguous [B,H,Lq,topk] {dt} tensor")
+    rc = lib().topk_attn_fwd_masked(_ptr(q), _ptr(k), _ptr(v), _ptr(out), B, H, Lq, Lk, d, int(topk), int(chunk),
+                                    int(bool(causal)), _ptr(kv_len), _ptr(mask_words), int(mask_batch_stride),
+                                    int(mask_head_stride), _dtype_code(q), _ptr(idx), _ptr(score), _stream(stream))
+    _check(rc, "topk_attn_fwd_masked")
 
 
 def topk_attn_fwd_host(q, k, v, out, topk: int, chunk: int = 1024, causal: bool = False, stream=None) -> None:
@@ -271,8 +314,19 @@ def topk_pool_trim() -> None:
 # convenience wrappers that allocate the outputs ---------------------------------------------
 
 def attention(q, k, v, topk: int, chunk: int = 1024, causal: bool = False, return_indices: bool = False,
-              stream=None):
+              stream=None, kv_len=None, mask=None):
+    """Top-k attention; kv_len ([B] int32) and mask (bool [B|1, H|1, Lq, Lk], True = valid) add Eq. 2's
+    general masks."""
     out = torch.empty_like(q)
+    if kv_len is not None or mask is not None:
+        B, H, Lq, _ = q.shape
+        idx = score = None
+        if return_indices:
+            idx = torch.empty(B, H, Lq, topk, dtype=torch.int32, device=q.device)
+            score = torch.empty(B, H, Lq, topk, dtype=torch.float32, device=q.device)
+        words, bs, hs = pack_mask(mask) if mask is not None else (None, 0, 0)
+        topk_attn_fwd_masked(q, k, v, out, topk, chunk, causal, kv_len, words, bs, hs, idx, score, stream)
+        return (out, idx, score) if return_indices else out
     if not return_indices:
         topk_attn_fwd(q, k, v, out, topk, chunk, causal, stream)
         return out

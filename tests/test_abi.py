@@ -46,7 +46,7 @@ def _attn(lib, **kw):
 
 @pytest.mark.parametrize("kw,code", [
     (dict(q=None), -1), (dict(out=None), -1), (dict(B=0), -1), (dict(Lk=-1), -1), (dict(topk=0), -1),
-    (dict(topk=9), -1), (dict(chunk=0), -1), (dict(causal=1, Lk=9, topk=2), -1), (dict(causal=2), -1),
+    (dict(topk=9), -1), (dict(chunk=0), -1), (dict(causal=1, Lq=9, topk=2), -1), (dict(causal=2), -1),
     (dict(dtype=7), -1), (dict(d=96), -2), (dict(dtype=0, d=48), -2), (dict(topk=600, Lk=1000), -2),
     (dict(q=24), -2),
 ])
@@ -120,3 +120,16 @@ def test_backward_scratch_is_linear_in_the_cache():
     f = T.topk_ffn_bwd_workspace_bytes
     assert 4096 * 512 * 20 <= f(4096, 1024, 65536, 512) <= 4096 * 512 * 20 + 65536 * 8 + 4096
     assert f(4096, 4096, 65536, 512) == 0 and attn(1024, 0) == 0
+
+
+def test_masked_attention_argument_errors(lib):
+    f = lib.topk_attn_fwd_masked
+
+    def call(causal=0, kv_len=None, mask=None, mbs=0, mhs=0, Lq=8, Lk=8):
+        return f(16, 16, 16, 16, 1, 1, Lq, Lk, 64, 4, 8, causal, kv_len, mask, mbs, mhs, 1, None, None, None)
+
+    assert call(mbs=-1, mask=16) == -1
+    assert call(mhs=-4, mask=16) == -1
+    assert call(causal=1, Lq=9) == -1
+    assert call(mask=18) == -2      # not 4-byte aligned
+    assert call(kv_len=17) == -2
