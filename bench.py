@@ -111,10 +111,36 @@ def workload(args):
     return w
 
 
+def valid_pairs(w) -> float | None:
+    """(query, key) pairs that Eq. 2's masks leave valid, over all heads; None without masks."""
+    if not (w.causal or w.kv_len or w.mask_p):
+        return None
+    import numpy as np
+
+    from paper_2106_06899_gb300 import workloads as W
+
+    kv, mask = W.mask_inputs(w)
+    i = np.arange(w.Lq)
+    lim = np.minimum(i + 1 + (w.Lk - w.Lq), w.Lk) if w.causal else np.full(w.Lq, w.Lk)
+    total = 0.0
+    for b in range(w.B):
+        lb = np.minimum(lim, int(kv[b])) if kv is not None else lim
+        if mask is None:
+            total += float(lb.sum())
+        else:
+            m = mask[b, 0].numpy() & (np.arange(w.Lk)[None, :] < lb[:, None])
+            total += float(m.sum())
+    return total * w.H
+
+
 def work_flops(w) -> float:
-    """Algorithmic score-GEMM FLOPs of one call (every score is computed, Sec. 5)."""
+    """Algorithmic score-GEMM FLOPs of one call (every score is computed, Sec. 5); under a mask only
+    the valid pairs count."""
     if w.kind == "ffn":
         return 2.0 * w.N * w.d_ff * w.d_model
+    pairs = valid_pairs(w)
+    if pairs is not None:
+        return 2.0 * pairs * w.d
     if w.causal:  # only unmasked pairs j <= i
         pairs = w.Lq * (w.Lq + 1) / 2
         return 2.0 * w.B * w.H * pairs * w.d
@@ -128,7 +154,7 @@ FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 def roofline(w, achieved, pk):
     """Roofline of the dominant kernel: the tcgen05 kernels against the measured bf16 tensor peak; the
     SIMT kernel (fp32 inputs, or k above the tensor path's 128) against the fp32 FMA rate."""
-    simt = w.kind == "attn" and (w.dtype == "f32" or w.topk > 128)
+    simt = w.kind == "attn" and (w.dtype == "f32" or w.topk > 128 or w.mask_p > 0)
     if simt:
         return {"bound": "alu", "achieved": achieved, "peak": FP32_FMA_TFLOPS, "unit": "TFLOP/s",
                 "frac": achieved / FP32_FMA_TFLOPS, "traffic": None,
@@ -197,6 +223,14 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------ oracle timing
+def oracle_masks(w):
+    """Eq. 2's masks of a workload in the oracle's form (numpy), or Nones."""
+    from paper_2106_06899_gb300 import workloads as W
+
+    kv, mask = W.mask_inputs(w)
+    return (None if kv is None else kv.numpy()), (None if mask is None else mask.numpy())
+
+
 def oracle_rate(w, seconds: float, inputs, seed_rows: int = 0):
     """Oracle tokens/s on a bounded sample of rows of the workload (same inputs, all host cores).
 
@@ -212,7 +246,8 @@ def oracle_rate(w, seconds: float, inputs, seed_rows: int = 0):
         if w.kind == "ffn":
             res = oracle.ffn(*inputs, w.topk, rows=rows)
         else:
-            res = oracle.topk_attention(*inputs, w.topk, causal=w.causal, rows=rows)
+            kv, mask = oracle_masks(w)
+            res = oracle.topk_attention(*inputs, w.topk, causal=w.causal, rows=rows, kv_len=kv, mask=mask)
         return rows, res, time.perf_counter() - t0
 
     rows, res, t = run(max(cores, 16))
@@ -235,13 +270,17 @@ def parity_check(w, host, dev, out, rows, ref):
     import oracle
     from oracle.parity import check_rows
     from paper_2106_06899_gb300 import topk as T
+    from paper_2106_06899_gb300 import workloads as W
 
     if w.kind == "ffn":
         _, idx, score = T.ffn(dev[0], dev[1], dev[2], w.topk, return_indices=True)
         q, k, v = (t[None, None] for t in host)
         act, dtype, d = oracle.RELU, "bf16", w.d_model
     else:
-        _, idx, score = T.attention(dev[0], dev[1], dev[2], w.topk, w.chunk, w.causal, return_indices=True)
+        kv, mask = W.mask_inputs(w)
+        _, idx, score = T.attention(dev[0], dev[1], dev[2], w.topk, w.chunk, w.causal, return_indices=True,
+                                    kv_len=None if kv is None else kv.cuda(),
+                                    mask=None if mask is None else mask.cuda())
         q, k, v = host
         act, dtype, d = oracle.SOFTMAX, w.dtype, w.d
     T.topk_check()
@@ -251,8 +290,9 @@ def parity_check(w, host, dev, out, rows, ref):
     gscore = score.reshape(-1, w.topk)[r].cpu().numpy()
     del idx, score
     try:
+        okv, omask = oracle_masks(w) if w.kind == "attn" else (None, None)
         st = check_rows(q=q, k=k, v=v, rows=rows, gpu_out=gout, gpu_idx=gidx, gpu_score=gscore, topk=w.topk,
-                        dtype=dtype, act=act, causal=w.causal, ref=ref)
+                        dtype=dtype, act=act, causal=w.causal, ref=ref, kv_len=okv, mask=omask)
         return {"ok": True, **st}
     except AssertionError as e:
         return {"ok": False, "rows": len(rows), "error": str(e)}
@@ -277,7 +317,8 @@ def run_reference(args):
         if w.kind == "ffn":
             oracle.ffn(*inputs, w.topk, rows=rows)
         else:
-            oracle.topk_attention(*inputs, w.topk, causal=w.causal, rows=rows)
+            kv, mask = oracle_masks(w)
+            oracle.topk_attention(*inputs, w.topk, causal=w.causal, rows=rows, kv_len=kv, mask=mask)
         return len(rows), time.perf_counter() - t0
 
     n, t = step(max(cores, 16), 0)
@@ -342,6 +383,7 @@ def run_ours(args):
     host = W.make_inputs(w.with_(seed=w.seed + rank))
     dev = [t.cuda() for t in host]
     in_bytes = sum(t.numel() * t.element_size() for t in host)
+    masked = False
     if w.kind == "ffn":
         out = torch.empty(w.N, w.d_model, dtype=torch.float32, device="cuda")
 
@@ -350,8 +392,17 @@ def run_ours(args):
     else:
         out = torch.empty_like(dev[0])
 
+        kv, mask = W.mask_inputs(w)
+        masked = kv is not None or mask is not None
+        dkv = None if kv is None else kv.cuda()
+        words, mbs, mhs = T.pack_mask(mask.cuda()) if mask is not None else (None, 0, 0)
+
         def step():
-            T.topk_attn_fwd(dev[0], dev[1], dev[2], out, w.topk, w.chunk, w.causal)
+            if masked:
+                T.topk_attn_fwd_masked(dev[0], dev[1], dev[2], out, w.topk, w.chunk, w.causal, dkv, words, mbs,
+                                       mhs)
+            else:
+                T.topk_attn_fwd(dev[0], dev[1], dev[2], out, w.topk, w.chunk, w.causal)
 
     flush = None
     if in_bytes <= 2 * L2_BYTES:
@@ -410,6 +461,21 @@ def run_ours(args):
         if w.kind == "ffn":
             def e2e_step():
                 T.topk_ffn_fwd_host(pinned[0], pinned[1], pinned[2], hout, w.topk)
+        elif masked:
+            # no host-buffer entry takes masks: the inputs are copied on the stream, then the masked call
+            # and the copy back, all through the public binding
+            hkv = None if kv is None else kv.pin_memory()
+            hmask = None if words is None else words.cpu().pin_memory()
+
+            def e2e_step():
+                dq_, dk_, dv_ = (t.to("cuda", non_blocking=True) for t in pinned)
+                dkv_ = None if hkv is None else hkv.to("cuda", non_blocking=True)
+                dm_ = None if hmask is None else hmask.to("cuda", non_blocking=True)
+                T.topk_attn_fwd_masked(dq_, dk_, dv_, out, w.topk, w.chunk, w.causal, dkv_, dm_, mbs, mhs)
+                hout.copy_(out, non_blocking=True)
+                torch.cuda.synchronize()
+
+            in_bytes += (0 if hkv is None else hkv.numel() * 4) + (0 if hmask is None else hmask.numel() * 4)
         else:
             def e2e_step():
                 T.topk_attn_fwd_host(pinned[0], pinned[1], pinned[2], hout, w.topk, w.chunk, w.causal)

@@ -50,6 +50,10 @@ class Workload:
     chunk: int = 0
     causal: bool = False
     dist: str = "normal"
+    # Eq. 2's general masks: key counts per batch (key padding), and the density of a random bit
+    # mask shared by the heads of a batch (0 = none)
+    kv_len: tuple = ()
+    mask_p: float = 0.0
     # feed-forward
     N: int = 0
     d_model: int = 0
@@ -81,7 +85,26 @@ WORKLOADS = {
                            d=128, chunk=2048, causal=True, note="causal decoder-style, d = 128"),
     "ffn_65k": Workload("ffn_65k", "ffn", "bf16", seed=4, topk=512, N=4096, d_model=1024, d_ff=65536,
                         dist="ffn", note="top-k feed-forward, T5-large-like d_ff = 65536"),
+    # Eq. 2's masks
+    "decode_65k": Workload("decode_65k", "attn", "bf16", seed=5, topk=64, B=4, H=12, Lq=128, Lk=65536, d=64,
+                           chunk=128, causal=True, dist="lowrank",
+                           note="the last 128 positions against a 65,536-key cache, causal"),
+    "bert_padded": Workload("bert_padded", "attn", "bf16", seed=6, topk=64, B=8, H=12, Lq=512, Lk=512, d=64,
+                            chunk=512, kv_len=(512, 500, 448, 400, 320, 256, 128, 64),
+                            note="BERT-base shape, batches padded to 512 keys"),
+    "bert_masked": Workload("bert_masked", "attn", "bf16", seed=7, topk=64, B=8, H=12, Lq=512, Lk=512, d=64,
+                            chunk=512, mask_p=0.5, note="BERT-base shape, random bit mask (half the pairs)"),
 }
+
+
+def mask_inputs(w: "Workload"):
+    """(kv_len int32 [B] or None, boolean mask [B, 1, Lq, Lk] or None) of a workload, seeded."""
+    kv = torch.tensor(w.kv_len, dtype=torch.int32) if w.kv_len else None
+    mask = None
+    if w.mask_p > 0:
+        g = torch.Generator().manual_seed(int(w.seed) + 999)
+        mask = torch.rand(w.B, 1, w.Lq, w.Lk, generator=g) < w.mask_p
+    return kv, mask
 
 
 def _torch_dtype(dtype: str) -> torch.dtype:
