@@ -142,6 +142,23 @@ int topk_attn_fwd_masked(const void* q, const void* k, const void* v, void* out,
                          float* score, void* stream);
 
 /*
+ * Plain (vanilla) attention, Eq. 1 (Sec. 2.1), under Eq. 2's causal mask and
+ * per-batch key counts: the softmax covers every valid key.  It is the path
+ * the paper compares top-k attention with (Sec. 3; query chunking, Sec. 2.2,
+ * bounds its memory there): here the score tile stays on chip, so no
+ * [chunk x Lk] buffer exists and `chunk` is validated but has no effect.
+ *   q, k, v, out, B, H, Lq, Lk, causal, kv_len: as topk_attn_fwd_masked.
+ *   d      : 64 or 128.  dtype: TOPK_BF16 only (fp32 is TOPK_ERR_UNSUPPORTED).
+ *   B * H  : at most 65535.
+ *   Scratch: topk_vanilla_attn_workspace_bytes() (V transposed, B*H*d*Lk*2
+ *   bytes rounded up), from the library's pool.  A row with no valid key
+ *   writes zeros.  Errors as topk_attn_fwd.
+ */
+int topk_vanilla_attn_fwd(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk,
+                          int d, int chunk, int causal, const int32_t* kv_len, int dtype, void* stream);
+size_t topk_vanilla_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, int dtype);
+
+/*
  * Top-k feed-forward layer, Eq. 3 with the top-k of Eq. 4 and ReLU as the
  * activation (Sec. 2.1, Sec. 2.2).
  *   x  : [N, d_model] bf16 device pointer (the queries).

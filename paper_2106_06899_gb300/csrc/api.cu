@@ -180,6 +180,19 @@ int run_ffn(FfnArgs a, cudaStream_t st) {
 
 size_t elem_bytes(int dtype) { return dtype == TOPK_F32 ? 4 : 2; }
 
+int validate_plain(const PlainArgs& a, int chunk, int dtype) {
+  if (!a.q || !a.k || !a.v || !a.out) return TOPK_ERR_INVALID_ARG;
+  if (a.B <= 0 || a.H <= 0 || a.Lq <= 0 || a.Lk <= 0 || a.d <= 0 || chunk < 1) return TOPK_ERR_INVALID_ARG;
+  if (a.causal != 0 && a.causal != 1) return TOPK_ERR_INVALID_ARG;
+  if (a.causal && a.Lq > a.Lk) return TOPK_ERR_INVALID_ARG;
+  if (dtype != TOPK_F32 && dtype != TOPK_BF16) return TOPK_ERR_INVALID_ARG;
+  if (dtype != TOPK_BF16 || (a.d != 64 && a.d != 128)) return TOPK_ERR_UNSUPPORTED;
+  if (static_cast<long long>(a.B) * a.H > 65535) return TOPK_ERR_UNSUPPORTED;
+  if (!aligned16(a.q) || !aligned16(a.k) || !aligned16(a.v) || !aligned16(a.out)) return TOPK_ERR_UNSUPPORTED;
+  if (a.kv_len && (reinterpret_cast<uintptr_t>(a.kv_len) & 3u)) return TOPK_ERR_UNSUPPORTED;
+  return TOPK_OK;
+}
+
 // Backward pass (bwd.cu): the cache width, the entry and bucket counts are
 // bounded so that slots and offsets fit in 32-bit integers.
 constexpr int kBwdMaxK = 2048;
@@ -304,6 +317,33 @@ int topk_ffn_fwd_indices(const void* x, const void* W1, const void* W2, void* ou
                          int topk, int32_t* idx, float* score, void* stream) {
   FfnArgs a{x, W1, W2, static_cast<float*>(out), N, d_model, d_ff, topk, idx, score, nullptr, 0};
   return run_ffn(a, static_cast<cudaStream_t>(stream));
+}
+
+int topk_vanilla_attn_fwd(const void* q, const void* k, const void* v, void* out, int B, int H, int Lq, int Lk,
+                          int d, int chunk, int causal, const int32_t* kv_len, int dtype, void* stream) {
+  PlainArgs a{q, k, v, out, B, H, Lq, Lk, d, causal, kv_len, nullptr};
+  int rc = validate_plain(a, chunk, dtype);
+  if (rc) return rc;
+  DeviceState* dev = device_state();
+  if (!dev) return TOPK_ERR_NO_DEVICE;
+  if (dev->cc_major != 10 || dev->cc_minor != 3) return TOPK_ERR_NO_DEVICE;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  void* buf = nullptr;
+  if (!pool_alloc(&buf, plain_workspace_bytes(B, H, Lk, d), st)) return TOPK_ERR_CUDA;
+  a.workspace = buf;
+  const int n = attn_plain(a, make_ctl(dev), dev->num_sms, st);
+  cudaFreeAsync(buf, st);
+  if (n == 0) return TOPK_ERR_UNSUPPORTED;
+  if (n < 0) return TOPK_ERR_CUDA;
+  t_last_launches = n;
+  return TOPK_OK;
+}
+
+size_t topk_vanilla_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, int dtype) {
+  PlainArgs a{reinterpret_cast<void*>(16), reinterpret_cast<void*>(16), reinterpret_cast<void*>(16),
+              reinterpret_cast<void*>(16), B, H, Lq, Lk, d, 0, nullptr, nullptr};
+  if (validate_plain(a, 1, dtype) != TOPK_OK) return 0;
+  return plain_workspace_bytes(B, H, Lk, d);
 }
 
 int topk_attn_bwd(const void* q, const void* k, const void* v, const void* dout, const int32_t* idx,

@@ -101,6 +101,20 @@ bool attn_bwd_supports(int d, int dtype);
 int attn_bwd(const AttnBwdArgs& a, int num_sms, cudaStream_t st);
 int ffn_bwd(const FfnBwdArgs& a, int num_sms, cudaStream_t st);
 
+// Plain attention (attn_plain.cu): Eq. 1 under the causal mask and key counts,
+// bf16, d in {64, 128}; the workspace holds V^T (plain_workspace_bytes).
+struct PlainArgs {
+  const void* q;
+  const void* k;
+  const void* v;
+  void* out;
+  int B, H, Lq, Lk, d, causal;
+  const int32_t* kv_len;
+  void* workspace;
+};
+size_t plain_workspace_bytes(int B, int H, int Lk, int d);
+int attn_plain(const PlainArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st);
+
 // Driver entry point for cuTensorMapEncodeTiled (resolved once, no libcuda link).
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                    const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,

@@ -51,6 +51,9 @@ def lib() -> ctypes.CDLL:
             L.topk_ffn_workspace_bytes.restype = sz
             L.topk_attn_fwd_masked.argtypes = [vp, vp, vp, vp] + [i32] * 8 + [vp, vp, ctypes.c_longlong,
                                                                             ctypes.c_longlong, i32, vp, vp, vp]
+            L.topk_vanilla_attn_fwd.argtypes = [vp, vp, vp, vp] + [i32] * 7 + [vp, i32, vp]
+            L.topk_vanilla_attn_workspace_bytes.argtypes = [i32] * 6
+            L.topk_vanilla_attn_workspace_bytes.restype = sz
             L.topk_attn_bwd.argtypes = [vp] * 9 + [i32] * 7 + [vp]
             L.topk_ffn_bwd.argtypes = [vp] * 9 + [i32] * 4 + [vp]
             L.topk_attn_bwd_workspace_bytes.argtypes = [i32] * 7
@@ -70,7 +73,7 @@ def lib() -> ctypes.CDLL:
                       "topk_attn_fwd_host", "topk_ffn_fwd_host", "topk_ffn_fwd_noalloc", "topk_check",
                       "topk_last_launch_count",
                       "topk_debug_skip_arrive", "topk_pool_usage", "topk_pool_trim", "topk_attn_bwd",
-                      "topk_ffn_bwd", "topk_attn_fwd_masked"):
+                      "topk_ffn_bwd", "topk_attn_fwd_masked", "topk_vanilla_attn_fwd"):
                 getattr(L, f).restype = i32
             _lib = L
     return _lib
@@ -177,6 +180,27 @@ def topk_attn_fwd_masked(q, k, v, out, topk: int, chunk: int = 1024, causal: boo
                                     int(bool(causal)), _ptr(kv_len), _ptr(mask_words), int(mask_batch_stride),
                                     int(mask_head_stride), _dtype_code(q), _ptr(idx), _ptr(score), _stream(stream))
     _check(rc, "topk_attn_fwd_masked")
+
+
+def topk_vanilla_attn_fwd(q, k, v, out, chunk: int = 1024, causal: bool = False, kv_len=None,
+                          stream=None) -> None:
+    """Plain attention (Eq. 1) over every valid key, the comparison path (bf16, d 64 or 128)."""
+    B, H, Lq, Lk, d = _attn_dims(q, k, v, out)
+    if kv_len is not None and (kv_len.dtype != torch.int32 or tuple(kv_len.shape) != (B,)):
+        raise ValueError("kv_len must be a [B] int32 tensor")
+    rc = lib().topk_vanilla_attn_fwd(_ptr(q), _ptr(k), _ptr(v), _ptr(out), B, H, Lq, Lk, d, int(chunk),
+                                     int(bool(causal)), _ptr(kv_len), _dtype_code(q), _stream(stream))
+    _check(rc, "topk_vanilla_attn_fwd")
+
+
+def topk_vanilla_attn_workspace_bytes(B, H, Lq, Lk, d, dtype) -> int:
+    return int(lib().topk_vanilla_attn_workspace_bytes(B, H, Lq, Lk, d, dtype))
+
+
+def vanilla_attention(q, k, v, chunk: int = 1024, causal: bool = False, kv_len=None, stream=None):
+    out = torch.empty_like(q)
+    topk_vanilla_attn_fwd(q, k, v, out, chunk, causal, kv_len, stream)
+    return out
 
 
 def topk_attn_fwd_host(q, k, v, out, topk: int, chunk: int = 1024, causal: bool = False, stream=None) -> None:

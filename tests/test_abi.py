@@ -133,3 +133,18 @@ def test_masked_attention_argument_errors(lib):
     assert call(causal=1, Lq=9) == -1
     assert call(mask=18) == -2      # not 4-byte aligned
     assert call(kv_len=17) == -2
+
+
+def test_vanilla_attention_argument_errors(lib):
+    f = lib.topk_vanilla_attn_fwd
+
+    def call(q=16, B=1, H=1, Lq=8, Lk=8, d=64, chunk=8, causal=0, kv_len=None, dtype=1):
+        return f(q, 16, 16, 16, B, H, Lq, Lk, d, chunk, causal, kv_len, dtype, None)
+
+    assert call(q=None) == -1 and call(Lk=0) == -1 and call(chunk=0) == -1 and call(dtype=3) == -1
+    assert call(causal=1, Lq=9) == -1
+    assert call(dtype=0) == -2 and call(d=96) == -2 and call(q=24) == -2
+    assert call(B=300, H=300) == -2  # more than 65535 (batch, head) problems
+    # scratch: V transposed, keys rounded up to a multiple of 8
+    assert T.topk_vanilla_attn_workspace_bytes(2, 3, 100, 1001, 64, 1) == 2 * 3 * 64 * 1008 * 2
+    assert T.topk_vanilla_attn_workspace_bytes(2, 3, 100, 1001, 64, 0) == 0

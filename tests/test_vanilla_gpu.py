@@ -1,0 +1,81 @@
+"""GPU parity of plain attention (Eq. 1 under Eq. 2's causal mask and key counts), the comparison
+path, through the C ABI against the oracle's plain attention (pinned against SDPA).
+
+The kernel rounds the softmax weights to bf16 before the P V product and writes bf16, so the
+bf16 output tolerance of the top-k path (2e-2) applies.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2106_06899_gb300 import topk as T
+from paper_2106_06899_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+TOL = 2e-2
+
+
+def _run(q, k, v, causal=False, kv_len=None):
+    kl = None if kv_len is None else torch.as_tensor(np.asarray(kv_len, np.int32)).cuda()
+    out = T.vanilla_attention(q.cuda(), k.cuda(), v.cuda(), causal=causal, kv_len=kl)
+    T.topk_check()
+    return out.float().cpu().numpy().reshape(-1, q.shape[-1])
+
+
+@pytest.mark.parametrize("B,H,Lq,Lk,d,causal", [
+    (2, 3, 300, 700, 64, False),
+    (1, 2, 257, 513, 128, False),
+    (1, 2, 640, 640, 64, True),
+    (2, 2, 7, 2048, 64, True),    # decode: the last 7 positions
+    (1, 1, 1, 1001, 128, True),   # one query; a key count that is not a multiple of 8
+    (3, 2, 129, 130, 64, False),  # ragged tiles on both sides
+])
+def test_vanilla_matches_oracle(B, H, Lq, Lk, d, causal):
+    q, k, v = W.attention_inputs(B, H, Lq, Lk, d, seed=100 + Lq)
+    got = _run(q, k, v, causal)
+    ref = oracle.vanilla(q, k, v, causal=causal)
+    err = np.abs(got - ref).max()
+    assert err <= TOL, err
+
+
+def test_vanilla_key_counts_and_empty_rows():
+    B, H, Lq, Lk, d = 4, 2, 200, 900, 64
+    q, k, v = W.attention_inputs(B, H, Lq, Lk, d, seed=110)
+    kv_len = [900, 333, 5, 0]
+    got = _run(q, k, v, kv_len=kv_len)
+    ref = oracle.vanilla(q, k, v, kv_len=kv_len)
+    assert np.abs(got - ref).max() <= TOL
+    assert np.all(got.reshape(B, H, Lq, d)[3] == 0)
+
+
+def test_vanilla_rescales_when_the_row_maximum_moves():
+    # scores grow along the keys, so each row's maximum rises tile after tile (and by more than the
+    # rescale margin): the running sum and O are rescaled many times
+    B, H, Lq, Lk, d = 1, 2, 256, 4096, 64
+    q, k, v = W.attention_inputs(B, H, Lq, Lk, d, dtype="f32", seed=111)
+    ramp = torch.linspace(0.2, 6.0, Lk)[None, None, :, None]
+    k = (k * ramp).to(torch.bfloat16)
+    q = (q * 2).to(torch.bfloat16)
+    v = v.to(torch.bfloat16)
+    got = _run(q, k, v)
+    ref = oracle.vanilla(q, k, v)
+    assert np.abs(got - ref).max() <= TOL
+
+
+def test_vanilla_equals_topk_with_every_key():
+    # k = Lk keeps every key: the top-k path (CUDA-core kernel at k = 512) and the plain path agree
+    w = W.WORKLOADS["bert_base_all_keys"]
+    q, k, v = W.make_inputs(w)
+    plain = _run(q, k, v)
+    topk = T.attention(q.cuda(), k.cuda(), v.cuda(), w.topk).float().cpu().numpy().reshape(-1, w.d)
+    assert np.abs(plain - topk).max() <= 2 * TOL
+
+
+def test_vanilla_long_65k_sampled_rows():
+    w = W.WORKLOADS["long_65k"].with_(H=2)
+    q, k, v = W.make_inputs(w)
+    got = _run(q, k, v)
+    rows = W.sample_rows(w.rows, 512, seed=7).numpy()
+    ref = oracle.vanilla(q, k, v, rows=rows)
+    assert np.abs(got[rows] - ref).max() <= TOL
