@@ -51,8 +51,10 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU work budget of the oracle baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-clocks", action="store_true")
-    p.add_argument("--pass", dest="which", choices=["fwd", "bwd"], default="fwd",
-                   help="bwd: time the backward pass (Sec. 2.2) for the forward pass's cache instead")
+    p.add_argument("--pass", dest="which", choices=["fwd", "bwd", "plain"], default="fwd",
+                   help="bwd: time the backward pass (Sec. 2.2) for the forward pass's cache instead; "
+                        "plain: the comparison path without top-k (Eq. 1 attention / the dense FF layer)")
+    p.add_argument("--ffn-chunk", type=int, default=16384, help="d_ff slice of the dense FF comparison path")
     p.add_argument("--kernel-only", action="store_true",
                    help="time the device call only: no end-to-end leg, clocks or CPU baseline (profiling)")
     a = p.parse_args()
@@ -653,12 +655,122 @@ def run_backward(args):
     print(json.dumps(line), flush=True)
 
 
+# ------------------------------------------------------------------ comparison path
+PLAIN_METRIC = "plain attention / dense FF tokens/s (comparison path, no top-k)"
+
+
+def run_plain(args):
+    """Times the path top-k is compared with (Sec. 3): plain attention over every valid key (Eq. 1)
+    or the dense FF layer (Eq. 3 without top-k), on the same workload, with the oracle's parity check
+    on sampled rows after the timed region."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2106_06899_gb300 import topk as T
+    from paper_2106_06899_gb300 import workloads as W
+
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    w = workload(args)
+    host = W.make_inputs(w)
+    dev = [t.cuda() for t in host]
+    if w.kind == "ffn":
+        out = torch.empty(w.N, w.d_model, dtype=torch.float32, device="cuda")
+
+        def step():
+            T.topk_vanilla_ffn_fwd(dev[0], dev[1], dev[2], out, args.ffn_chunk)
+
+        flops = 4.0 * w.N * w.d_ff * w.d_model
+        kernel = "cuBLAS GEMMs + relu_bf16_kernel"
+    else:
+        kv, _ = W.mask_inputs(w)
+        dkv = None if kv is None else kv.cuda()
+        out = torch.empty_like(dev[0])
+
+        def step():
+            T.topk_vanilla_attn_fwd(dev[0], dev[1], dev[2], out, w.chunk, w.causal, dkv)
+
+        pairs = valid_pairs(w.with_(mask_p=0.0))
+        flops = 4.0 * w.d * (pairs if pairs is not None else w.B * w.H * w.Lq * w.Lk)
+        kernel = "attn_plain_kernel"
+    flush = torch.empty(2 * L2_BYTES // 4, dtype=torch.float32, device="cuda")
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        step()
+    T.topk_check()
+    launches = T.topk_last_launch_count()
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(0).uuid)
+    except Exception:
+        pass
+    sampler = ClockSampler(uuid)
+    if not args.no_clocks:
+        sampler.start()
+        time.sleep(0.3)
+    torch.cuda.synchronize()
+    tot = 0.0
+    for _ in range(args.steps):
+        flush.fill_(1.0)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        tot += e0.elapsed_time(e1)
+    ms = tot / args.steps
+    clocks = None if args.no_clocks else sampler.stop()
+    T.topk_check()
+    pk = peaks()
+    achieved = flops / (ms / 1e3) / 1e12
+    line = {
+        "metric": PLAIN_METRIC, "value": w.tokens / (ms / 1e3), "unit": "tokens/s", "n_gpus": 1,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {**config_dict(w, "L2 flushed between steps (write of 2x L2 size)"),
+                   **({"ffn_chunk": args.ffn_chunk} if w.kind == "ffn" else {})},
+        "tflops": achieved,
+        "roofline": {"bound": "tensor", "achieved": achieved, "peak": pk["bf16"], "unit": "TFLOP/s",
+                     "frac": achieved / pk["bf16"], "traffic": None,
+                     "peak_source": f"{pk['source']} bf16 dense (burst)", "kernel": kernel,
+                     "flops": "4 d per valid (query, key) pair: S = QK^T and O = PV" if w.kind == "attn"
+                     else "4 d_model per (token, key): both GEMMs"},
+        "gpu_launches": launches * args.steps, "clocks": clocks, "e2e": None,
+    }
+    # parity on sampled rows against the oracle's plain attention / dense FF
+    rows = W.sample_rows(w.rows, 256, seed=3).numpy()
+    t0 = time.perf_counter()
+    if w.kind == "ffn":
+        ref = oracle.ffn_dense(*host, rows=rows)
+        t = time.perf_counter() - t0
+        got = out.cpu().numpy()[rows]
+        # H = ReLU(x W1^T) is rounded to bf16 before the second product: an element may be off by
+        # 2^-9 sum_j H_j |W2_j| (the dense layer on |W2|) plus the fp32 sums
+        bound = 2.0 ** -8 * oracle.ffn_dense(host[0], host[1], host[2].abs(), rows=rows) + 1e-5
+    else:
+        okv, _ = oracle_masks(w.with_(mask_p=0.0))
+        ref = oracle.vanilla(*host, causal=w.causal, rows=rows, kv_len=okv)
+        t = time.perf_counter() - t0
+        got = out.float().reshape(-1, w.d).cpu().numpy()[rows]
+        bound = np.full(got.shape, 2e-2)
+    err = float(np.abs(got - ref).max())
+    line["parity"] = {"ok": bool(np.all(np.abs(got - ref) <= bound)), "rows": len(rows), "max_err": err}
+    per_token = w.H if w.kind == "attn" else 1
+    line["cpu_baseline"] = {"value": len(rows) / per_token / t, "unit": "tokens/s", "cores": oracle.hardware_threads(),
+                            "kind": "oracle", "sample": f"{len(rows)} of {w.rows} rows, fp64 oracle, {t:.1f} s"}
+    print(json.dumps(line), flush=True)
+    if not line["parity"]["ok"]:
+        sys.exit(f"parity check of the plain path failed: max error {err}")
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
         run_reference(args)
     elif args.which == "bwd":
         run_backward(args)
+    elif args.which == "plain":
+        run_plain(args)
     else:
         run_ours(args)
 

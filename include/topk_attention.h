@@ -159,6 +159,21 @@ int topk_vanilla_attn_fwd(const void* q, const void* k, const void* v, void* out
 size_t topk_vanilla_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, int dtype);
 
 /*
+ * The dense feed-forward layer, Eq. 3 without top-k (Sec. 2.1): out =
+ * ReLU(x W1^T) W2, the comparison path for topk_ffn_fwd (Sec. 3).  d_ff is
+ * taken in slices of `chunk` keys (chunking bounds the memory, Sec. 2.2): per
+ * slice the hidden activations [N, chunk] are formed in bf16, ReLU'd and
+ * multiplied into the fp32 output.  The two products run in cuBLAS (plain
+ * GEMMs, bf16 inputs, fp32 accumulation); ReLU in the library's own kernel.
+ *   x, W1, W2, out, N, d_model, d_ff: as topk_ffn_fwd (d_model a multiple of 8).
+ *   chunk  : keys per slice, >= 1; a multiple of 8 unless it covers all of d_ff.
+ *   Scratch: topk_vanilla_ffn_workspace_bytes() = N * min(chunk, d_ff) * 2 bytes.
+ */
+int topk_vanilla_ffn_fwd(const void* x, const void* W1, const void* W2, void* out, int N, int d_model, int d_ff,
+                         int chunk, void* stream);
+size_t topk_vanilla_ffn_workspace_bytes(int N, int d_model, int d_ff, int chunk);
+
+/*
  * Top-k feed-forward layer, Eq. 3 with the top-k of Eq. 4 and ReLU as the
  * activation (Sec. 2.1, Sec. 2.2).
  *   x  : [N, d_model] bf16 device pointer (the queries).

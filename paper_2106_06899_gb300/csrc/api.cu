@@ -346,6 +346,45 @@ size_t topk_vanilla_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, in
   return plain_workspace_bytes(B, H, Lk, d);
 }
 
+namespace {
+int validate_ffn_plain(const FfnPlainArgs& a) {
+  if (!a.x || !a.W1 || !a.W2 || !a.out) return TOPK_ERR_INVALID_ARG;
+  if (a.N <= 0 || a.d_model <= 0 || a.d_ff <= 0 || a.chunk < 1) return TOPK_ERR_INVALID_ARG;
+  if (a.d_model % 8 != 0) return TOPK_ERR_UNSUPPORTED;
+  const long long c = a.chunk < a.d_ff ? a.chunk : a.d_ff;
+  if (c % 8 != 0 && c != a.d_ff) return TOPK_ERR_UNSUPPORTED;  // H rows stay 16-byte aligned
+  if ((static_cast<long long>(a.N) * c) % 8 != 0) return TOPK_ERR_UNSUPPORTED;
+  if (!aligned16(a.x) || !aligned16(a.W1) || !aligned16(a.W2) || !aligned16(a.out)) return TOPK_ERR_UNSUPPORTED;
+  return TOPK_OK;
+}
+}  // namespace
+
+int topk_vanilla_ffn_fwd(const void* x, const void* W1, const void* W2, void* out, int N, int d_model, int d_ff,
+                         int chunk, void* stream) {
+  FfnPlainArgs a{x, W1, W2, static_cast<float*>(out), N, d_model, d_ff, chunk, nullptr};
+  int rc = validate_ffn_plain(a);
+  if (rc) return rc;
+  DeviceState* dev = device_state();
+  if (!dev) return TOPK_ERR_NO_DEVICE;
+  if (dev->cc_major != 10 || dev->cc_minor != 3) return TOPK_ERR_NO_DEVICE;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  void* buf = nullptr;
+  if (!pool_alloc(&buf, ffn_plain_workspace_bytes(N, d_ff, chunk), st)) return TOPK_ERR_CUDA;
+  a.workspace = buf;
+  const int n = ffn_plain(a, dev->num_sms, st);
+  cudaFreeAsync(buf, st);
+  if (n <= 0) return TOPK_ERR_CUDA;
+  t_last_launches = n;
+  return TOPK_OK;
+}
+
+size_t topk_vanilla_ffn_workspace_bytes(int N, int d_model, int d_ff, int chunk) {
+  FfnPlainArgs a{reinterpret_cast<void*>(16), reinterpret_cast<void*>(16), reinterpret_cast<void*>(16),
+                 reinterpret_cast<float*>(16), N, d_model, d_ff, chunk, nullptr};
+  if (validate_ffn_plain(a) != TOPK_OK) return 0;
+  return ffn_plain_workspace_bytes(N, d_ff, chunk);
+}
+
 int topk_attn_bwd(const void* q, const void* k, const void* v, const void* dout, const int32_t* idx,
                   const float* score, float* dq, float* dk, float* dv, int B, int H, int Lq, int Lk, int d,
                   int topk, int dtype, void* stream) {

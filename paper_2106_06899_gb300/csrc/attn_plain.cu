@@ -7,8 +7,8 @@
 // registers: per 128-query tile and 128-key tile,
 //   S = Q K^T          tcgen05.mma into one of two TMEM score buffers;
 //   P = exp(S - m)     four softmax warps, one query row per thread, written
-//                      as bf16 into shared memory in the layout the next MMA
-//                      reads (128-byte swizzled, K-major);
+//                      as bf16 into one of two shared-memory buffers in the
+//                      layout the next MMA reads (128-byte swizzled, K-major);
 //   O += P V           tcgen05.mma into a TMEM accumulator of d columns, with
 //                      V read as its transpose V^T [d, L_K] (made once per call
 //                      by a transpose kernel) so that both MMAs take K-major
@@ -36,15 +36,15 @@ struct PlainLayout {
   static constexpr uint32_t Q_BYTES = BM * D * 2;
   static constexpr uint32_t K_BYTES = BN * D * 2;  // a key tile, keys x d
   static constexpr uint32_t V_BYTES = D * BN * 2;  // the same keys of V^T, d x keys (two 64-key blocks)
-  static constexpr uint32_t P_BYTES = BM * BN * 2;
+  static constexpr uint32_t P_BYTES = BM * BN * 2;  // one of two P buffers
   static constexpr size_t OFF_Q = 0;
   static constexpr size_t OFF_K = OFF_Q + Q_BYTES;
   static constexpr size_t OFF_V = OFF_K + static_cast<size_t>(S) * K_BYTES;
   static constexpr size_t OFF_P = OFF_V + static_cast<size_t>(S) * V_BYTES;
-  static constexpr size_t OFF_BAR = OFF_P + P_BYTES;
+  static constexpr size_t OFF_BAR = OFF_P + 2 * static_cast<size_t>(P_BYTES);
   // full/empty per K/V stage, q full/empty, s full/empty per score buffer,
-  // p_full, pv_done, o_empty, drain
-  static constexpr int NBARS = 2 * S + 2 + 4 + 4;
+  // p_full/pv_done per P buffer, o_empty, drain
+  static constexpr int NBARS = 2 * S + 2 + 4 + 4 + 2;
   static constexpr size_t BYTES = 1024 + OFF_BAR + NBARS * 8 + 16;
   static constexpr uint32_t TMEM_COLS = 512;
   static constexpr uint32_t O_COL = 2 * BN;  // O after the two score buffers
@@ -96,6 +96,15 @@ __device__ __forceinline__ void fence_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
+constexpr float kLog2e = 1.4426950408889634f;  // log2(e)
+
+// 2^x by the hardware approximation (ex2.approx); 2^-inf = 0
+__device__ __forceinline__ float ex2_approx(float x) {
+  float r;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&h);
@@ -124,10 +133,10 @@ __global__ void __launch_bounds__(192, 1)
   uint64_t* q_empty = bars + 2 * S + 1;
   uint64_t* s_full = bars + 2 * S + 2;   // [2]
   uint64_t* s_empty = bars + 2 * S + 4;  // [2]
-  uint64_t* p_full = bars + 2 * S + 6;
-  uint64_t* pv_done = bars + 2 * S + 7;
-  uint64_t* o_empty = bars + 2 * S + 8;
-  uint64_t* drain = bars + 2 * S + 9;
+  uint64_t* p_full = bars + 2 * S + 6;   // [2]
+  uint64_t* pv_done = bars + 2 * S + 8;  // [2]
+  uint64_t* o_empty = bars + 2 * S + 10;
+  uint64_t* drain = bars + 2 * S + 11;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + L::NBARS);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
@@ -144,8 +153,10 @@ __global__ void __launch_bounds__(192, 1)
       mbar_init(&s_full[b], 1);
       mbar_init(&s_empty[b], 4);
     }
-    mbar_init(p_full, 4);
-    mbar_init(pv_done, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&p_full[b], 4);
+      mbar_init(&pv_done[b], 1);
+    }
     mbar_init(o_empty, 4);
     mbar_init(drain, 1);
     *abort_flag = 0;
@@ -225,9 +236,9 @@ __global__ void __launch_bounds__(192, 1)
     // ------------------------------------------------------------ MMA issuer
     uint32_t it = 0, sc = 0, pc = 0, qi = 0;
     bool ok = true;
-    auto issue_pv = [&](uint32_t stage, bool first) {
+    auto issue_pv = [&](uint32_t stage, uint32_t pb, bool first) {
       const uint32_t o_tmem = tmem_base + L::O_COL;
-      const uint32_t pa = smem_u32(p_s);
+      const uint32_t pa = smem_u32(p_s + static_cast<size_t>(pb) * L::P_BYTES);
       const uint32_t va = smem_u32(v_s + static_cast<size_t>(stage) * L::V_BYTES);
 #pragma unroll
       for (int st = 0; st < BN / 16; ++st) {
@@ -235,7 +246,7 @@ __global__ void __launch_bounds__(192, 1)
         mma_bf16_ss(o_tmem, sdesc_k128(pa + r * BM * 128 + off), sdesc_k128(va + r * D * 128 + off), IDESC_O,
                     (first && st == 0) ? 0u : 1u);
       }
-      mma_commit(pv_done);
+      mma_commit(&pv_done[pb]);
       mma_commit(&empty_kv[stage]);
     };
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x, ++qi) {
@@ -277,12 +288,13 @@ __global__ void __launch_bounds__(192, 1)
             ok = false;
             break;
           }
-          if (!warp_wait_p(p_full, pc & 1u, ctl, abort_flag)) {
+          // P number pc sits in buffer pc & 1, that buffer's (pc >> 1)-th use
+          if (!warp_wait_p(&p_full[pc & 1u], (pc >> 1) & 1u, ctl, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          if (lane == 0) issue_pv(prev_stage, kt == 1);
+          if (lane == 0) issue_pv(prev_stage, pc & 1u, kt == 1);
           __syncwarp();
           ++pc;
         }
@@ -315,6 +327,7 @@ __global__ void __launch_bounds__(192, 1)
       const int i_row = qt * BM + row;
       const int nk = key_tiles(bh, qt);
       const int lim = min(kv_end(bh), causal ? min(i_row + 1 + coff, Lk) : Lk);  // keys j < lim are valid
+      const int lim_min = min(kv_end(bh), causal ? min(qt * BM + 1 + coff, Lk) : Lk);  // smallest in the tile
       float m_run = -INFINITY, z = 0.f;
       for (int kt = 0; kt < nk; ++kt, ++sc) {
         const int b = sc & 1u;
@@ -332,70 +345,87 @@ __global__ void __launch_bounds__(192, 1)
         __syncwarp();
         if (lane == 0) mbar_arrive(&s_empty[b]);
         const int j0 = kt * BN;
-        float mt = -INFINITY;
+        if (j0 + BN > lim_min) {  // only tiles that reach past some row's limit need the mask
 #pragma unroll
-        for (int e = 0; e < BN; ++e) {
-          if (j0 + e >= lim) s[e] = -INFINITY;
-          mt = fmaxf(mt, s[e]);
+          for (int e = 0; e < BN; ++e)
+            if (j0 + e >= lim) s[e] = -INFINITY;
         }
+        float mt = s[0];
+#pragma unroll
+        for (int e = 1; e + 1 < BN; e += 2) mt = max3f(mt, s[e], s[e + 1]);
+        mt = fmaxf(mt, s[BN - 1]);
         const bool raise = mt > m_run + kRescale || (m_run == -INFINITY && mt > -INFINITY);
         const float m_new = raise ? mt : m_run;
-        const float alpha = (raise && m_run > -INFINITY) ? __expf(m_run - m_new) : 1.f;
-        // P (and O) of the previous key tile must have been consumed
-        if (kt > 0) {
-          if (!warp_wait_p(pv_done, pc & 1u, ctl, abort_flag)) {
+        const float alpha = (raise && m_run > -INFINITY) ? ex2_approx((m_run - m_new) * kLog2e) : 1.f;
+        m_run = m_new;
+        // P row as packed bf16, computed before any wait on the previous products:
+        // exp(s - m) = 2^(s log2(e) - m log2(e)); a row with no valid key so far has p = 0
+        uint32_t w[BN / 2];
+        float zp[4] = {0.f, 0.f, 0.f, 0.f};  // four partial sums: no long dependent chain
+        if (m_run == -INFINITY) {
+#pragma unroll
+          for (int e = 0; e < BN / 2; ++e) w[e] = 0u;
+        } else {
+          const float ml = m_run * kLog2e;
+#pragma unroll
+          for (int e = 0; e < BN / 2; ++e) {
+            const float p0 = ex2_approx(fmaf(s[2 * e], kLog2e, -ml));
+            const float p1 = ex2_approx(fmaf(s[2 * e + 1], kLog2e, -ml));
+            w[e] = pack_bf16x2(p0, p1);
+            zp[e & 3] += p0 + p1;
+          }
+        }
+        const float zt = (zp[0] + zp[1]) + (zp[2] + zp[3]);
+        z = z * alpha + zt;
+        // P number pc goes to buffer pc & 1, whose previous P (number pc - 2) its product must have read;
+        // a rescale of O needs the previous product (number pc - 1) done as well
+        const uint32_t pb = pc & 1u;
+        if (pc >= 2 && !warp_wait_p(&pv_done[pb], ((pc - 2) >> 1) & 1u, ctl, abort_flag)) {
+          ok = false;
+          break;
+        }
+        if (kt > 0 && __any_sync(0xffffffffu, alpha != 1.f)) {
+          if (!warp_wait_p(&pv_done[(pc - 1) & 1u], ((pc - 1) >> 1) & 1u, ctl, abort_flag)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          ++pc;
-          if (__any_sync(0xffffffffu, alpha != 1.f)) {
 #pragma unroll 1
-            for (int c = 0; c < D; c += 32) {
-              float o[32];
-              tmem_ld32(o_taddr + c, o);
-              tmem_wait_ld();
+          for (int c = 0; c < D; c += 32) {
+            float o[32];
+            tmem_ld32(o_taddr + c, o);
+            tmem_wait_ld();
 #pragma unroll
-              for (int e = 0; e < 32; ++e) o[e] *= alpha;
-              tmem_st32(o_taddr + c, o);
-            }
-            tmem_wait_st();
+            for (int e = 0; e < 32; ++e) o[e] *= alpha;
+            tmem_st32(o_taddr + c, o);
           }
+          tmem_wait_st();
         }
-        z *= alpha;
-        m_run = m_new;
-        // P row as bf16, 128-byte swizzled K-major: row `row` of block r holds keys 64r .. 64r + 63,
-        // its 16-byte chunk c at chunk position c ^ (row & 7)
+        // 128-byte swizzled K-major: row `row` of block r holds keys 64r .. 64r + 63, its 16-byte
+        // chunk c at chunk position c ^ (row & 7)
+        uint8_t* pbuf = p_s + static_cast<size_t>(pb) * L::P_BYTES;
 #pragma unroll
         for (int r = 0; r < 2; ++r) {
-          uint8_t* prow = p_s + r * BM * 128 + row * 128;
+          uint8_t* prow = pbuf + r * BM * 128 + row * 128;
 #pragma unroll
           for (int c = 0; c < 8; ++c) {
-            uint32_t w[4];
-#pragma unroll
-            for (int h = 0; h < 4; ++h) {
-              const int e = r * 64 + c * 8 + 2 * h;
-              const float p0 = m_run == -INFINITY ? 0.f : __expf(s[e] - m_run);
-              const float p1 = m_run == -INFINITY ? 0.f : __expf(s[e + 1] - m_run);
-              w[h] = pack_bf16x2(p0, p1);
-              z += __uint_as_float(w[h] << 16) + __uint_as_float(w[h] & 0xffff0000u);
-            }
-            *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) << 4)) = make_uint4(w[0], w[1], w[2], w[3]);
+            const int e = r * 32 + c * 4;
+            *reinterpret_cast<uint4*>(prow + ((c ^ (row & 7)) << 4)) = make_uint4(w[e], w[e + 1], w[e + 2], w[e + 3]);
           }
         }
         fence_async_smem();  // the MMA (async proxy) reads what these generic stores wrote
         tc_fence_before();   // and the rescaled O above
         __syncwarp();
-        if (lane == 0) mbar_arrive(p_full);
+        if (lane == 0) mbar_arrive(&p_full[pb]);
+        ++pc;
       }
       if (!ok) break;
-      // the last tile's P V, then out = O / z
-      if (!warp_wait_p(pv_done, pc & 1u, ctl, abort_flag)) {
+      // the last tile's P V (number pc - 1; products complete in issue order), then out = O / z
+      if (!warp_wait_p(&pv_done[(pc - 1) & 1u], ((pc - 1) >> 1) & 1u, ctl, abort_flag)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      ++pc;
       const float inv = z > 0.f ? 1.f / z : 0.f;
 #pragma unroll 1
       for (int c = 0; c < D; c += 32) {

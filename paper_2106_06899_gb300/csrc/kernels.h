@@ -115,6 +115,19 @@ struct PlainArgs {
 size_t plain_workspace_bytes(int B, int H, int Lk, int d);
 int attn_plain(const PlainArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st);
 
+// Dense FF (ffn_plain.cu): ReLU(x W1^T) W2 in d_ff slices of `chunk` keys, the
+// two products in cuBLAS; the workspace holds one slice of H (bf16).
+struct FfnPlainArgs {
+  const void* x;
+  const void* W1;
+  const void* W2;
+  float* out;
+  int N, d_model, d_ff, chunk;
+  void* workspace;
+};
+size_t ffn_plain_workspace_bytes(int N, int d_ff, int chunk);
+int ffn_plain(const FfnPlainArgs& a, int num_sms, cudaStream_t st);
+
 // Driver entry point for cuTensorMapEncodeTiled (resolved once, no libcuda link).
 using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                    const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,

@@ -54,6 +54,9 @@ def lib() -> ctypes.CDLL:
             L.topk_vanilla_attn_fwd.argtypes = [vp, vp, vp, vp] + [i32] * 7 + [vp, i32, vp]
             L.topk_vanilla_attn_workspace_bytes.argtypes = [i32] * 6
             L.topk_vanilla_attn_workspace_bytes.restype = sz
+            L.topk_vanilla_ffn_fwd.argtypes = [vp, vp, vp, vp] + [i32] * 4 + [vp]
+            L.topk_vanilla_ffn_workspace_bytes.argtypes = [i32] * 4
+            L.topk_vanilla_ffn_workspace_bytes.restype = sz
             L.topk_attn_bwd.argtypes = [vp] * 9 + [i32] * 7 + [vp]
             L.topk_ffn_bwd.argtypes = [vp] * 9 + [i32] * 4 + [vp]
             L.topk_attn_bwd_workspace_bytes.argtypes = [i32] * 7
@@ -73,7 +76,7 @@ def lib() -> ctypes.CDLL:
                       "topk_attn_fwd_host", "topk_ffn_fwd_host", "topk_ffn_fwd_noalloc", "topk_check",
                       "topk_last_launch_count",
                       "topk_debug_skip_arrive", "topk_pool_usage", "topk_pool_trim", "topk_attn_bwd",
-                      "topk_ffn_bwd", "topk_attn_fwd_masked", "topk_vanilla_attn_fwd"):
+                      "topk_ffn_bwd", "topk_attn_fwd_masked", "topk_vanilla_attn_fwd", "topk_vanilla_ffn_fwd"):
                 getattr(L, f).restype = i32
             _lib = L
     return _lib
@@ -200,6 +203,23 @@ def topk_vanilla_attn_workspace_bytes(B, H, Lq, Lk, d, dtype) -> int:
 def vanilla_attention(q, k, v, chunk: int = 1024, causal: bool = False, kv_len=None, stream=None):
     out = torch.empty_like(q)
     topk_vanilla_attn_fwd(q, k, v, out, chunk, causal, kv_len, stream)
+    return out
+
+
+def topk_vanilla_ffn_fwd(x, W1, W2, out, chunk: int = 16384, stream=None) -> None:
+    """The dense FF layer (Eq. 3 without top-k) in d_ff slices of `chunk` keys: out fp32 [N, d_model]."""
+    N, dm, dff = _ffn_dims(x, W1, W2, out)
+    rc = lib().topk_vanilla_ffn_fwd(_ptr(x), _ptr(W1), _ptr(W2), _ptr(out), N, dm, dff, int(chunk), _stream(stream))
+    _check(rc, "topk_vanilla_ffn_fwd")
+
+
+def topk_vanilla_ffn_workspace_bytes(N, d_model, d_ff, chunk) -> int:
+    return int(lib().topk_vanilla_ffn_workspace_bytes(N, d_model, d_ff, chunk))
+
+
+def vanilla_ffn(x, W1, W2, chunk: int = 16384, stream=None):
+    out = torch.empty(x.shape[0], x.shape[1], dtype=torch.float32, device=x.device)
+    topk_vanilla_ffn_fwd(x, W1, W2, out, chunk, stream)
     return out
 
 

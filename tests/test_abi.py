@@ -148,3 +148,14 @@ def test_vanilla_attention_argument_errors(lib):
     # scratch: V transposed, keys rounded up to a multiple of 8
     assert T.topk_vanilla_attn_workspace_bytes(2, 3, 100, 1001, 64, 1) == 2 * 3 * 64 * 1008 * 2
     assert T.topk_vanilla_attn_workspace_bytes(2, 3, 100, 1001, 64, 0) == 0
+
+
+def test_dense_ffn_argument_errors(lib):
+    f = lib.topk_vanilla_ffn_fwd
+    assert f(None, 16, 16, 16, 4, 64, 128, 64, None) == -1
+    assert f(16, 16, 16, 16, 4, 64, 128, 0, None) == -1
+    assert f(16, 16, 16, 16, 4, 60, 128, 64, None) == -2   # d_model not a multiple of 8
+    assert f(16, 16, 16, 16, 4, 64, 128, 60, None) == -2   # slice not a multiple of 8
+    assert f(24, 16, 16, 16, 4, 64, 128, 64, None) == -2
+    assert T.topk_vanilla_ffn_workspace_bytes(4096, 1024, 65536, 16384) == 4096 * 16384 * 2
+    assert T.topk_vanilla_ffn_workspace_bytes(4096, 1024, 1000, 16384) == 4096 * 1000 * 2

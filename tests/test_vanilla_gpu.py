@@ -79,3 +79,34 @@ def test_vanilla_long_65k_sampled_rows():
     rows = W.sample_rows(w.rows, 512, seed=7).numpy()
     ref = oracle.vanilla(q, k, v, rows=rows)
     assert np.abs(got[rows] - ref).max() <= TOL
+
+
+@pytest.mark.parametrize("N,dm,dff,chunk", [
+    (333, 256, 4096, 1024),
+    (128, 1024, 65536, 16384),
+    (200, 512, 3000, 1024),   # a last slice of 952 keys
+    (64, 192, 700, 700),      # one slice
+])
+def test_dense_ffn_matches_oracle(N, dm, dff, chunk):
+    # the hidden activations H = ReLU(x W1^T) are rounded to bf16 (relative error 2^-9) before the
+    # second product, so an output element can be off by up to 2^-9 sum_j H_j |W2_j| plus the fp32
+    # sums; that sum is the dense layer applied to |W2| (the oracle's, exact)
+    x, w1, w2 = W.ffn_inputs(N, dm, dff, seed=120 + N)
+    out = T.vanilla_ffn(x.cuda(), w1.cuda(), w2.cuda(), chunk)
+    T.topk_check()
+    ref = oracle.ffn_dense(x, w1, w2)
+    scale = oracle.ffn_dense(x, w1, w2.abs())
+    err = np.abs(out.cpu().numpy() - ref)
+    assert np.all(err <= 2.0 ** -8 * scale + 1e-5), float((err / (2.0 ** -8 * scale + 1e-5)).max())
+
+
+def test_dense_ffn_equals_topk_ffn_with_every_key():
+    # k = d_ff keeps every key: both paths compute the dense layer (each within its own bound)
+    N, dm, dff = 96, 256, 1024
+    x, w1, w2 = W.ffn_inputs(N, dm, dff, seed=130)
+    dense = T.vanilla_ffn(x.cuda(), w1.cuda(), w2.cuda(), 512).cpu().numpy()
+    topk = T.ffn(x.cuda(), w1.cuda(), w2.cuda(), dff).cpu().numpy()
+    ref = oracle.ffn_dense(x, w1, w2)
+    scale = oracle.ffn_dense(x, w1, w2.abs())
+    assert np.all(np.abs(dense - ref) <= 2.0 ** -8 * scale + 1e-5)
+    assert np.abs(topk - ref).max() <= TOL
