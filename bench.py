@@ -51,7 +51,7 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU work budget of the oracle baseline")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--no-clocks", action="store_true")
-    p.add_argument("--pass", dest="which", choices=["fwd", "bwd", "plain"], default="fwd",
+    p.add_argument("--pass", dest="which", choices=["fwd", "bwd", "plain", "decoder"], default="fwd",
                    help="bwd: time the backward pass (Sec. 2.2) for the forward pass's cache instead; "
                         "plain: the comparison path without top-k (Eq. 1 attention / the dense FF layer)")
     p.add_argument("--ffn-chunk", type=int, default=16384, help="d_ff slice of the dense FF comparison path")
@@ -763,6 +763,62 @@ def run_plain(args):
         sys.exit(f"parity check of the plain path failed: max error {err}")
 
 
+# ------------------------------------------------------------------ decoder composition
+DECODER_METRIC = "12-layer decoder training step tokens/s (top-k attention, Sec. 3)"
+
+
+def run_decoder(args):
+    """Forward + backward of the 12-layer decoder (d_model 768, 12 heads, d_ff 3072, top-64 causal
+    attention, dense FF) over one sequence of L tokens (--L, default 32768): time per step and peak
+    device memory (PyTorch's allocator plus the library's pool)."""
+    import torch
+
+    from paper_2106_06899_gb300 import topk as T
+    from paper_2106_06899_gb300.decoder import Decoder
+
+    torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+    L = args.L or 32768
+    torch.manual_seed(0)
+    results = {}
+    for name, topk in (("top64", 64), ("plain_sdpa", None)):
+        model = Decoder(12, 768, 12, 3072, topk=topk, ffn_topk=None)
+        x = torch.randn(1, L, 768, device="cuda", dtype=torch.bfloat16)
+
+        def step():
+            for p in model.parameters():
+                p.grad = None
+            model(x).float().pow(2).mean().backward()
+
+        try:
+            for _ in range(max(args.warmup, 1)):
+                step()
+            torch.cuda.synchronize()
+            torch.cuda.reset_peak_memory_stats()
+            T.topk_pool_usage(reset_high=True)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(args.steps):
+                step()
+            e1.record()
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1) / args.steps
+            pool_hi, _ = T.topk_pool_usage()
+            results[name] = {"ms_per_step": ms, "tokens_per_s": L / (ms / 1e3),
+                             "peak_torch_bytes": torch.cuda.max_memory_allocated(), "peak_library_pool_bytes": pool_hi}
+        except torch.OutOfMemoryError:
+            results[name] = {"error": "out of device memory"}
+        del model, x
+        torch.cuda.empty_cache()
+    top = results["top64"]
+    line = {"metric": DECODER_METRIC, "value": top.get("tokens_per_s"), "unit": "tokens/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": top.get("ms_per_step"),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "decoder", "layers": 12, "d_model": 768, "heads": 12, "d_ff": 3072, "L": L,
+                       "topk": 64, "ffn": "dense", "attention_backward": "cached kept set (Sec. 2.2)"},
+            "runs": results, "e2e": None}
+    print(json.dumps(line), flush=True)
+
+
 def main():
     args = parse_args()
     if args.impl == "reference":
@@ -771,6 +827,8 @@ def main():
         run_backward(args)
     elif args.which == "plain":
         run_plain(args)
+    elif args.which == "decoder":
+        run_decoder(args)
     else:
         run_ours(args)
 
