@@ -232,7 +232,8 @@ int topk_attn_bwd(const void* q, const void* k, const void* v, const void* dout,
  *   idx, score: [N, topk] int32 / fp32 device, the cache.
  *   dx        : [N, d_model] fp32; dW1, dW2: [d_ff, d_model] fp32 (written).
  *   d_model   : a multiple of 64, at most 2048.  1 <= topk <= d_ff.
- *   Scratch: topk_ffn_bwd_workspace_bytes().  Errors as topk_ffn_fwd.
+ *   Scratch: topk_ffn_bwd_workspace_bytes() (20 bytes per cache entry, 4 more per
+ *   cache entry and 256 columns of d_model, 8 per key).  Errors as topk_ffn_fwd.
  */
 int topk_ffn_bwd(const void* x, const void* W1, const void* W2, const float* dout, const int32_t* idx,
                  const float* score, float* dx, float* dW1, float* dW2, int N, int d_model, int d_ff, int topk,

@@ -401,7 +401,7 @@ int topk_ffn_bwd(const void* x, const void* W1, const void* W2, const float* dou
                  void* stream) {
   FfnBwdArgs a{x, W1, W2, dout, idx, score, dx, dW1, dW2, N, d_model, d_ff, topk, nullptr};
   return run_bwd(
-      a, validate_ffn_bwd(a), [](const FfnBwdArgs& y) { return ffn_bwd_workspace_bytes(y.N, y.d_ff, y.topk); },
+      a, validate_ffn_bwd(a), [](const FfnBwdArgs& y) { return ffn_bwd_workspace_bytes(y.N, y.d_model, y.d_ff, y.topk); },
       [](const FfnBwdArgs& y, int sms, cudaStream_t s) { return ffn_bwd(y, sms, s); },
       static_cast<cudaStream_t>(stream));
 }
@@ -419,7 +419,7 @@ size_t topk_ffn_bwd_workspace_bytes(int N, int d_model, int d_ff, int topk) {
   float* f = reinterpret_cast<float*>(16);
   FfnBwdArgs a{p, p, p, f, reinterpret_cast<const int32_t*>(16), f, f, f, f, N, d_model, d_ff, topk, nullptr};
   if (validate_ffn_bwd(a) != TOPK_OK) return 0;
-  return ffn_bwd_workspace_bytes(N, d_ff, topk);
+  return ffn_bwd_workspace_bytes(N, d_model, d_ff, topk);
 }
 
 size_t topk_attn_workspace_bytes(int B, int H, int Lq, int Lk, int d, int topk, int chunk, int dtype) {

@@ -15,7 +15,8 @@
 //             atomic count per key; the count it saw is its slot);
 //   2. scan:  bucket offsets, the exclusive prefix sum of the counts;
 //   3. rows:  per query row the steps above up to dq_i; each entry
-//             (i, ds_t, a_t, j_t) is written to its bucket slot;
+//             (i, ds_t, a_t, j_t) is written to its bucket slot (the FF layer
+//             reads its long W1/W2 rows in column chunks, chunk-major);
 //   4. keys:  the entry list, now grouped by key, is cut into equal runs of
 //             entries; a lane group walks its run, adds ds q_i into dk_j and
 //             a dout_i into dv_j in registers, and writes a key's sums when
@@ -329,95 +330,123 @@ __global__ void __launch_bounds__(kRowWarps * 32) attn_bwd_rows_kernel(
 }
 
 // ---------------------------------------------------------------------------
-// 3b. rows, the ReLU feed-forward layer.  One CTA per token; its 8 warps take
-// the kept entries t = w, w + 8, ...; lane l reads the 16-byte chunks l,
-// l + 32, ... of a W1/W2 row (CPL chunks: d_model <= 256 CPL).  ReLU's
-// backward needs no other entry of the row, so da_t, ds_t and the dx term
-// come from one pass.  The warps' dx partial sums meet in shared memory.
-template <int CPL>
-__global__ void __launch_bounds__(kRowWarps * 32) ffn_bwd_rows_kernel(
-    const __nv_bfloat16* __restrict__ W1, const __nv_bfloat16* __restrict__ W2, const float* __restrict__ dout,
-    const int32_t* __restrict__ idx, const float* __restrict__ score, const int* __restrict__ rank,
-    const int* __restrict__ off, BwdEntry* __restrict__ ent, float* __restrict__ dx, int N, int DM, int dff,
-    int K) {
-  extern __shared__ float red[];  // [kRowWarps][DM]
+// 3b. rows, the ReLU feed-forward layer, in column chunks of kFfChunk.  A
+// token's k rows of W2 (and of W1) are 2 KB each at d_model = 1024 and W1 and
+// W2 together exceed L2, so the rows are read chunk-major: all tokens read
+// their rows' first kFfChunk columns before any reads the next chunk, and the
+// columns in use (d_ff x kFfChunk bf16, 32 MB at d_ff = 65536) stay in L2.
+//   da:  per (chunk, token) a warp per kept entry sums dout_i . W2_j over the
+//        chunk's columns (one 16-byte vector per lane, a warp sum) into
+//        part[chunk][token][t];
+//   dx:  per (chunk, token) ds_t = sum over chunks of part (0 unless s_t > 0,
+//        ReLU's backward), then dx_i = sum_t ds_t W1_{j_t} over the chunk's
+//        columns (each thread 4 columns, 8 rows in flight); the chunk-0 CTA
+//        of a token also writes its entries to their key buckets.
+constexpr int kFfChunk = 256;
+constexpr int kDaWarps = 8;
+constexpr int kDxThreads = kFfChunk / 4;
+
+__global__ void __launch_bounds__(kDaWarps * 32) ffn_bwd_da_kernel(
+    const __nv_bfloat16* __restrict__ W2, const float* __restrict__ dout, const int32_t* __restrict__ idx,
+    const float* __restrict__ score, float* __restrict__ part, int N, int DM, int dff, int K) {
+  const int i = blockIdx.x % N, chunk = blockIdx.x / N;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nch = DM / 8;
-  for (int i = blockIdx.x; i < N; i += gridDim.x) {
-    float go[CPL][8], acc[CPL][8];
+  const int col = chunk * kFfChunk + lane * 8;
+  const bool live = col < DM;
+  float g[8];
+  if (live)
+    load_f32<8>(dout + static_cast<long long>(i) * DM + col, g);
+  else
 #pragma unroll
-    for (int u = 0; u < CPL; ++u) {
-      const int ch = lane + 32 * u;
+    for (int e = 0; e < 8; ++e) g[e] = 0.f;
+  const int32_t* ki = idx + static_cast<long long>(i) * K;
+  const float* ks = score + static_cast<long long>(i) * K;
+  float* out = part + (static_cast<long long>(chunk) * N + i) * K;
+  constexpr int U = 4;  // kept entries in flight per warp
+  for (int t0 = warp * U; t0 < K; t0 += kDaWarps * U) {
+    float f[U][8];
+    bool use[U];
 #pragma unroll
-      for (int e = 0; e < 8; ++e) acc[u][e] = 0.f;
-      if (ch < nch)
-        load_f32<8>(dout + static_cast<long long>(i) * DM + ch * 8, go[u]);
+    for (int u = 0; u < U; ++u) {
+      const int t = t0 + u;
+      const int j = t < K ? ki[t] : -1;
+      use[u] = t < K && j >= 0 && j < dff && ks[t] > 0.f;
+      if (use[u] && live)
+        Chunk<__nv_bfloat16>::load(W2 + static_cast<long long>(j) * DM + col, f[u]);
       else
 #pragma unroll
-        for (int e = 0; e < 8; ++e) go[u][e] = 0.f;
+        for (int e = 0; e < 8; ++e) f[u][e] = 0.f;
     }
-    for (int t = warp; t < K; t += kRowWarps) {
-      const int j = idx[static_cast<long long>(i) * K + t];
-      const float s = score[static_cast<long long>(i) * K + t];
-      if (j < 0 || j >= dff || !(s > 0.f)) continue;  // ReLU: a_t = ds_t = 0
-      const __nv_bfloat16* w2r = W2 + static_cast<long long>(j) * DM;
-      const __nv_bfloat16* w1r = W1 + static_cast<long long>(j) * DM;
-      float w1f[CPL][8];
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
       float p = 0.f;
 #pragma unroll
-      for (int u = 0; u < CPL; ++u) {
-        const int ch = lane + 32 * u;
-        if (ch < nch) {
-          float f[8];
-          Chunk<__nv_bfloat16>::load(w2r + ch * 8, f);
-          Chunk<__nv_bfloat16>::load(w1r + ch * 8, w1f[u]);
-#pragma unroll
-          for (int e = 0; e < 8; ++e) p = fmaf(f[e], go[u][e], p);
-        } else {
-#pragma unroll
-          for (int e = 0; e < 8; ++e) w1f[u][e] = 0.f;
-        }
-      }
-      const float ds = warp_sum(p);  // da_t; s_t > 0 so ds_t = da_t
-#pragma unroll
-      for (int u = 0; u < CPL; ++u)
-#pragma unroll
-        for (int e = 0; e < 8; ++e) acc[u][e] = fmaf(ds, w1f[u][e], acc[u][e]);
-      if (lane == 0) {
-        BwdEntry en;
-        en.row = i;
-        en.ds = ds;
-        en.a = s;
-        en.key = j;
-        ent[off[j] + rank[static_cast<long long>(i) * K + t]] = en;
-      }
+      for (int e = 0; e < 8; ++e) p = fmaf(f[u][e], g[e], p);
+      p = warp_sum(p);
+      if (lane == 0 && t0 + u < K) out[t0 + u] = use[u] ? p : 0.f;
     }
-    float* mine = red + static_cast<size_t>(warp) * DM;
-#pragma unroll
-    for (int u = 0; u < CPL; ++u) {
-      const int ch = lane + 32 * u;
-      if (ch < nch) {
-        float4* dst = reinterpret_cast<float4*>(mine + ch * 8);
-        dst[0] = make_float4(acc[u][0], acc[u][1], acc[u][2], acc[u][3]);
-        dst[1] = make_float4(acc[u][4], acc[u][5], acc[u][6], acc[u][7]);
-      }
-    }
-    __syncthreads();
-    for (int col = threadIdx.x; col < DM; col += blockDim.x) {
-      float s = 0.f;
-#pragma unroll
-      for (int w = 0; w < kRowWarps; ++w) s += red[w * DM + col];
-      dx[static_cast<long long>(i) * DM + col] = s;
-    }
-    __syncthreads();
   }
+}
+
+__global__ void __launch_bounds__(kDxThreads) ffn_bwd_dx_kernel(
+    const __nv_bfloat16* __restrict__ W1, const int32_t* __restrict__ idx, const float* __restrict__ score,
+    const float* __restrict__ part, const int* __restrict__ rank, const int* __restrict__ off,
+    BwdEntry* __restrict__ ent, float* __restrict__ dx, int N, int DM, int dff, int K, int nchunks) {
+  extern __shared__ float dsv[];  // [K] ds_t, then [K] key indices (as int)
+  int* jv = reinterpret_cast<int*>(dsv + K);
+  const int i = blockIdx.x % N, chunk = blockIdx.x / N;
+  const int tid = threadIdx.x;
+  for (int t = tid; t < K; t += kDxThreads) {
+    const int j = idx[static_cast<long long>(i) * K + t];
+    const float s = score[static_cast<long long>(i) * K + t];
+    const bool use = j >= 0 && j < dff && s > 0.f;
+    float ds = 0.f;
+    if (use)
+      for (int c = 0; c < nchunks; ++c) ds += part[(static_cast<long long>(c) * N + i) * K + t];
+    dsv[t] = ds;
+    jv[t] = use ? j : -1;
+    if (chunk == 0 && use) {  // this token's entries go to their key buckets once
+      BwdEntry en;
+      en.row = i;
+      en.ds = ds;
+      en.a = s;
+      en.key = j;
+      ent[off[j] + rank[static_cast<long long>(i) * K + t]] = en;
+    }
+  }
+  __syncthreads();
+  const int c0 = chunk * kFfChunk + tid * 4;
+  if (c0 >= DM) return;
+  float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+  for (int t0 = 0; t0 < K; t0 += 8) {
+    uint2 raw[8];
+    float w[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int t = t0 + u;
+      const int j = t < K ? jv[t] : -1;
+      w[u] = j >= 0 ? dsv[t] : 0.f;
+      raw[u] = j >= 0 ? __ldg(reinterpret_cast<const uint2*>(W1 + static_cast<long long>(j) * DM + c0))
+                      : make_uint2(0u, 0u);
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      a0 = fmaf(w[u], __uint_as_float(raw[u].x << 16), a0);
+      a1 = fmaf(w[u], __uint_as_float(raw[u].x & 0xffff0000u), a1);
+      a2 = fmaf(w[u], __uint_as_float(raw[u].y << 16), a2);
+      a3 = fmaf(w[u], __uint_as_float(raw[u].y & 0xffff0000u), a3);
+    }
+  }
+  *reinterpret_cast<float4*>(dx + static_cast<long long>(i) * DM + c0) = make_float4(a0, a1, a2, a3);
 }
 
 // ---------------------------------------------------------------------------
 // 4. keys.  The entry list is grouped by bucket (one bucket per key of each
 // (b, h)).  Lane groups of LPR lanes each take a run of kRun consecutive
 // entries; lane c of a group covers the 16-byte chunks c, c + LPR, ... (CPL
-// of them) of a q (or x) row and the same columns of dout.  A bucket's sums
+// of them) of a q (or x) row and the same columns of dout, within the column
+// slice of its grid row (blockIdx.y; the FF layer's 2 KB rows are split into
+// 256-column slices).  A bucket's sums
 // are written when its entries end inside the run: stored when the run
 // holds all of them, added atomically when they continue past either end of
 // the run.  U entries are loaded ahead so that their row reads overlap.
@@ -435,6 +464,7 @@ __global__ void __launch_bounds__(kKeyWarps * 32) bwd_keys_kernel(
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int grp = lane / LPR, c = lane % LPR;
   const int nch = D / VEC;
+  const int ch0 = blockIdx.y * LPR * CPL;  // the column slice of this grid row
   const long long E = *total_ptr;
   const long long n_runs = (E + kRun - 1) / kRun;
   const long long stride = static_cast<long long>(gridDim.x) * kKeyWarps * G;
@@ -452,7 +482,7 @@ __global__ void __launch_bounds__(kKeyWarps * 32) bwd_keys_kernel(
     auto flush = [&](bool partial) {
 #pragma unroll
       for (int u = 0; u < CPL; ++u) {
-        const int ch = c + LPR * u;
+        const int ch = ch0 + c + LPR * u;
         if (ch < nch) {
           float4* pk = reinterpret_cast<float4*>(dk + static_cast<long long>(cur) * D + ch * VEC);
           float4* pv = reinterpret_cast<float4*>(dv + static_cast<long long>(cur) * D + ch * VEC);
@@ -482,7 +512,7 @@ __global__ void __launch_bounds__(kKeyWarps * 32) bwd_keys_kernel(
         en[i] = ok ? ent[e0 + i] : BwdEntry{0, 0.f, 0.f, -1};
 #pragma unroll
         for (int u = 0; u < CPL; ++u) {
-          const int ch = c + LPR * u;
+          const int ch = ch0 + c + LPR * u;
           if (ok && ch < nch) {
             Chunk<T>::load(q + static_cast<long long>(en[i].row) * D + ch * VEC, fq[i][u]);
             load_cols<TD, VEC>(dout + static_cast<long long>(en[i].row) * D + ch * VEC, fg[i][u]);
@@ -532,14 +562,15 @@ struct BwdScratch {
   int* bsum;
   int* rank;
   BwdEntry* ent;
+  float* part;  // FF only: per column chunk, token and kept entry, the partial dout . W2_j
 };
 
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
 
-size_t scratch_bytes(long long n_buckets, long long n_entries) {
+size_t scratch_bytes(long long n_buckets, long long n_entries, long long n_part = 0) {
   const long long n_tiles = (n_buckets + kScanTile - 1) / kScanTile;
   return align256(n_buckets * 4) + align256((n_buckets + 1) * 4) + align256(n_tiles * 4) +
-         align256(n_entries * 4) + align256(n_entries * sizeof(BwdEntry));
+         align256(n_entries * 4) + align256(n_entries * sizeof(BwdEntry)) + align256(n_part * 4);
 }
 
 BwdScratch carve(void* ws, long long n_buckets, long long n_entries) {
@@ -555,6 +586,8 @@ BwdScratch carve(void* ws, long long n_buckets, long long n_entries) {
   s.rank = reinterpret_cast<int*>(p);
   p += align256(n_entries * 4);
   s.ent = reinterpret_cast<BwdEntry*>(p);
+  p += align256(n_entries * sizeof(BwdEntry));
+  s.part = reinterpret_cast<float*>(p);
   return s;
 }
 
@@ -571,13 +604,15 @@ int rank_and_scan(const BwdScratch& s, const int32_t* idx, const float* score, l
   return cudaGetLastError() == cudaSuccess ? 4 : -1;
 }
 
+// slices > 1 splits each row into column slices of LPR * CPL 16-byte chunks,
+// one grid row per slice: lighter lane groups, more of them in flight
 template <typename T, typename TD, int LPR, int CPL>
 int launch_keys(const T* q, const TD* dout, const BwdScratch& s, long long n_buckets, long long max_entries,
-                float* dk, float* dv, int D, int num_sms, cudaStream_t st) {
+                float* dk, float* dv, int D, int num_sms, cudaStream_t st, int slices = 1) {
   constexpr int G = 32 / LPR;
   const long long runs = (max_entries + kRun - 1) / kRun;
-  bwd_keys_kernel<T, TD, LPR, CPL><<<grid_for(runs, kKeyWarps * G, num_sms, 8), kKeyWarps * 32, 0, st>>>(
-      q, dout, s.ent, s.off + n_buckets, dk, dv, D);
+  const dim3 grid(grid_for(runs, kKeyWarps * G, num_sms, 8), slices);
+  bwd_keys_kernel<T, TD, LPR, CPL><<<grid, kKeyWarps * 32, 0, st>>>(q, dout, s.ent, s.off + n_buckets, dk, dv, D);
   return cudaGetLastError() == cudaSuccess ? 1 : -1;
 }
 
@@ -611,7 +646,6 @@ int attn_bwd_t(const AttnBwdArgs& a, int num_sms, cudaStream_t st) {
   return nk < 0 ? -1 : n + nk;
 }
 
-template <int CPL>
 int ffn_bwd_t(const FfnBwdArgs& a, int num_sms, cudaStream_t st) {
   const long long n_entries = static_cast<long long>(a.N) * a.topk;
   const long long n_buckets = a.d_ff;
@@ -624,17 +658,17 @@ int ffn_bwd_t(const FfnBwdArgs& a, int num_sms, cudaStream_t st) {
     return -1;
   int n = rank_and_scan(s, a.idx, a.score, n_entries, a.topk, a.N, a.d_ff, n_buckets, 1, num_sms, st);
   if (n < 0) return -1;
-  const size_t smem = static_cast<size_t>(kRowWarps) * a.d_model * sizeof(float);
-  auto rows = ffn_bwd_rows_kernel<CPL>;
-  if (smem > 48 * 1024 &&
-      cudaFuncSetAttribute(rows, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) != cudaSuccess)
-    return -1;
-  rows<<<grid_for(a.N, 1, num_sms, 4), kRowWarps * 32, smem, st>>>(W1, W2, a.dout, a.idx, a.score, s.rank, s.off,
-                                                                    s.ent, a.dx, a.N, a.d_model, a.d_ff, a.topk);
+  const int nchunks = (a.d_model + kFfChunk - 1) / kFfChunk;
+  const unsigned grid = static_cast<unsigned>(nchunks) * static_cast<unsigned>(a.N);
+  ffn_bwd_da_kernel<<<grid, kDaWarps * 32, 0, st>>>(W2, a.dout, a.idx, a.score, s.part, a.N, a.d_model, a.d_ff,
+                                                    a.topk);
+  const size_t smem = static_cast<size_t>(a.topk) * 8;
+  ffn_bwd_dx_kernel<<<grid, kDxThreads, smem, st>>>(W1, a.idx, a.score, s.part, s.rank, s.off, s.ent, a.dx, a.N,
+                                                    a.d_model, a.d_ff, a.topk, nchunks);
   if (cudaGetLastError() != cudaSuccess) return -1;
-  n += 1;
-  const int nk = launch_keys<__nv_bfloat16, float, 32, CPL>(x, a.dout, s, n_buckets, n_entries, a.dW1, a.dW2,
-                                                             a.d_model, num_sms, st);
+  n += 2;
+  const int nk = launch_keys<__nv_bfloat16, float, 32, 1>(x, a.dout, s, n_buckets, n_entries, a.dW1, a.dW2,
+                                                           a.d_model, num_sms, st, nchunks);
   return nk < 0 ? -1 : n + nk;
 }
 
@@ -645,8 +679,9 @@ size_t attn_bwd_workspace_bytes(int B, int H, int Lq, int Lk, int topk) {
   return scratch_bytes(static_cast<long long>(B) * H * Lk, R * topk);
 }
 
-size_t ffn_bwd_workspace_bytes(int N, int d_ff, int topk) {
-  return scratch_bytes(d_ff, static_cast<long long>(N) * topk);
+size_t ffn_bwd_workspace_bytes(int N, int d_model, int d_ff, int topk) {
+  const long long nchunks = (d_model + kFfChunk - 1) / kFfChunk;
+  return scratch_bytes(d_ff, static_cast<long long>(N) * topk, nchunks * N * topk);
 }
 
 bool attn_bwd_supports(int d, int dtype) {
@@ -670,12 +705,7 @@ int attn_bwd(const AttnBwdArgs& a, int num_sms, cudaStream_t st) {
 }
 
 int ffn_bwd(const FfnBwdArgs& a, int num_sms, cudaStream_t st) {
-  const int cpl = (a.d_model / 8 + 31) / 32;  // 16-byte chunks per lane
-  if (cpl <= 1) return ffn_bwd_t<1>(a, num_sms, st);
-  if (cpl <= 2) return ffn_bwd_t<2>(a, num_sms, st);
-  if (cpl <= 4) return ffn_bwd_t<4>(a, num_sms, st);
-  if (cpl <= 8) return ffn_bwd_t<8>(a, num_sms, st);
-  return 0;
+  return ffn_bwd_t(a, num_sms, st);
 }
 
 }  // namespace topk

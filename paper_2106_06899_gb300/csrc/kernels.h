@@ -96,7 +96,7 @@ struct FfnBwdArgs {
 };
 
 size_t attn_bwd_workspace_bytes(int B, int H, int Lq, int Lk, int topk);
-size_t ffn_bwd_workspace_bytes(int N, int d_ff, int topk);
+size_t ffn_bwd_workspace_bytes(int N, int d_model, int d_ff, int topk);
 bool attn_bwd_supports(int d, int dtype);
 int attn_bwd(const AttnBwdArgs& a, int num_sms, cudaStream_t st);
 int ffn_bwd(const FfnBwdArgs& a, int num_sms, cudaStream_t st);
