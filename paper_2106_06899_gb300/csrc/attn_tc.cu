@@ -34,6 +34,8 @@
 //
 // Every pipeline wait is bounded (common.cuh); on expiry the CTA stops,
 // drains its in-flight copies and MMAs, frees TMEM and returns.
+#include <algorithm>
+
 #include "kernels.h"
 #include "select.cuh"
 
@@ -191,7 +193,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmk,
                    const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ out, int BH, int H, int Lq,
                    int Lk, int topk, int rec_cap, int causal, const int32_t* __restrict__ kv_len, int n_units,
-                   int32_t* __restrict__ idx,
+                   int parts, uint64_t* __restrict__ part_keys, int* __restrict__ part_n, int32_t* __restrict__ idx,
                    float* __restrict__ score, uint64_t* __restrict__ park, int* __restrict__ park_n, DevCtl ctl) {
   using L = Layout<D, FK, SPLIT>;
   using Sel = typename L::Sel;
@@ -249,7 +251,13 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
   const uint32_t tmem_base = *tmem_slot;
 
   const int n_qt = (Lq + BM - 1) / BM;
-  auto decode = [&](int u, int& bh, int& qt) {
+  // A unit is (b, h, query tile, key part): with parts > 1 (grids that would
+  // leave SMs idle, as decoding a few positions against a long cache does)
+  // each query tile's key tiles are split into `parts` ranges, each part keeps
+  // its own top k, and a merge kernel combines them.
+  auto decode = [&](int u_, int& bh, int& qt, int& part) {
+    part = u_ % parts;
+    const int u = u_ / parts;
     if (causal) {  // heaviest query tiles first
       qt = n_qt - 1 - u / BH;
       bh = u % BH;
@@ -275,6 +283,18 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
   auto tile_limit_min = [&](int bh, int qt) {  // the smallest row limit of query tile qt
     return min(kv_end(bh), causal ? min(qt * BM + 1 + coff, Lk) : Lk);
   };
+  // key tiles [t0, t1) of a unit's part; a part left without tiles streams one
+  // fully masked tile (empty = true) so that every stage keeps its handshakes
+  auto tile_range = [&](int bh, int qt, int part, int& t0, int& t1, bool& empty) {
+    const int nk = key_tiles(bh, qt);
+    t0 = static_cast<int>(static_cast<long long>(part) * nk / parts);
+    t1 = static_cast<int>(static_cast<long long>(part + 1) * nk / parts);
+    empty = t1 <= t0;
+    if (empty) {
+      t0 = 0;
+      t1 = 1;
+    }
+  };
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -285,8 +305,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     uint32_t it = 0, q_issued = 0;
     bool ok = true;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-      int bh, qt;
-      decode(u, bh, qt);
+      int bh, qt, part;
+      decode(u, bh, qt, part);
       if (!warp_wait(q_empty, (q_issued & 1u) ^ 1u, ctl, abort_flag)) {
         ok = false;
         break;
@@ -296,8 +316,10 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         for (int r = 0; r < R; ++r) tma_load_3d(q_s + r * BM * 128, &tmq, q_full, r * 64, qt * BM, bh);
       }
       ++q_issued;
-      const int nk = key_tiles(bh, qt);
-      for (int kt = 0; kt < nk; ++kt) {
+      int t0, t1;
+      bool empty;
+      tile_range(bh, qt, part, t0, t1, empty);
+      for (int kt = t0; kt < t1; ++kt) {
         const int s = it % S;
         const uint32_t ph = (it / S) & 1u;
         if (!warp_wait(&empty_k[s], ph ^ 1u, ctl, abort_flag)) {
@@ -332,15 +354,17 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     uint32_t it = 0, acc_it = 0, qi = 0;
     bool ok = true;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x, ++qi) {
-      int bh, qt;
-      decode(u, bh, qt);
+      int bh, qt, part;
+      decode(u, bh, qt, part);
       if (!warp_wait(q_full, qi & 1u, ctl, abort_flag)) {
         ok = false;
         break;
       }
       tc_fence_after();
-      const int nk = key_tiles(bh, qt);
-      for (int kt = 0; kt < nk; ++kt, ++it, ++acc_it) {
+      int t0, t1;
+      bool empty;
+      tile_range(bh, qt, part, t0, t1, empty);
+      for (int kt = t0; kt < t1; ++kt, ++it, ++acc_it) {
         const int s = it % S;
         if (!warp_wait(&full_k[s], (it / S) & 1u, ctl, abort_flag)) {
           ok = false;
@@ -388,14 +412,16 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     f.init(ring_mem, row, rec_cap);
     bool ok = true;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-      int bh, qt;
-      decode(u, bh, qt);
+      int bh, qt, part;
+      decode(u, bh, qt, part);
       f.begin_unit();
       const int i_row = qt * BM + row;
-      const int nk = key_tiles(bh, qt);
-      const uint32_t lim = row_limit(bh, i_row);
-      const int lim_min = tile_limit_min(bh, qt);
-      for (int kt = 0; ok && kt < nk; ++kt, ++acc_it) {
+      int t0, t1;
+      bool empty;
+      tile_range(bh, qt, part, t0, t1, empty);
+      const uint32_t lim = empty ? 0u : row_limit(bh, i_row);
+      const int lim_min = empty ? 0 : tile_limit_min(bh, qt);
+      for (int kt = t0; ok && kt < t1; ++kt, ++acc_it) {
         const int b = acc_it % NACC;
         if (!warp_wait(&acc_full[b], (acc_it / NACC) & 1u, ctl, abort_flag)) {
           ok = false;
@@ -465,8 +491,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     const size_t park0 = (static_cast<size_t>(blockIdx.x) * 4 + quad) * 2;  // this warp's first slot
     uint32_t s = 0;                                                           // units done by this warp
     for (int u = blockIdx.x; u < n_units; u += gridDim.x, ++s) {
-      int bh, qt;
-      decode(u, bh, qt);
+      int bh, qt, part;
+      decode(u, bh, qt, part);
       const int i_row = qt * BM + row;
       heap.begin_unit(sel_mem, row, topk);
       // batch threshold: two thirds of the ring, within the filter's margin
@@ -498,8 +524,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     uint32_t s = 0;
     bool ok = true;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x, ++s) {
-      int bh, qt;
-      decode(u, bh, qt);
+      int bh, qt, part;
+      decode(u, bh, qt, part);
       for (int h = 0; h < 2; ++h) {
         const int q = 2 * e + h;
         if (!wait_count(&pk_done[q], s + 1, ctl, abort_flag)) {
@@ -512,7 +538,13 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         if (i_row < Lq) {  // a row without a valid key (n = 0) gets zeros
           const size_t orow = static_cast<size_t>(bh) * Lq + i_row;
           const ParkedKeys kept{park + slot * topk * 32 + lane, n};
-          softmax_gather_store<__nv_bfloat16, D>(kept, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
+          if (parts > 1) {  // this part's kept keys, for the merge
+            const size_t prow = static_cast<size_t>(part) * BH * Lq + orow;
+            for (int t = 0; t < n; ++t) part_keys[prow * topk + t] = kept.get(t);
+            part_n[prow] = n;
+          } else {
+            softmax_gather_store<__nv_bfloat16, D>(kept, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
+          }
         }
         __syncwarp();
         st_release_u32(&ep_done[q], s + 1);
@@ -527,14 +559,16 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     Sel heap;
     bool ok = true;
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
-      int bh, qt;
-      decode(u, bh, qt);
+      int bh, qt, part;
+      decode(u, bh, qt, part);
       const int i_row = qt * BM + row;
       heap.init(sel_mem, row, topk, rec_cap);
-      const int nk = key_tiles(bh, qt);
-      const uint32_t lim = row_limit(bh, i_row);
-      const int lim_min = tile_limit_min(bh, qt);
-      for (int kt = 0; kt < nk; ++kt, ++acc_it) {
+      int t0, t1;
+      bool empty;
+      tile_range(bh, qt, part, t0, t1, empty);
+      const uint32_t lim = empty ? 0u : row_limit(bh, i_row);
+      const int lim_min = empty ? 0 : tile_limit_min(bh, qt);
+      for (int kt = t0; kt < t1; ++kt, ++acc_it) {
         const int b = acc_it % NACC;
         if (!warp_wait(&acc_full[b], (acc_it / NACC) & 1u, ctl, abort_flag)) {
           ok = false;
@@ -564,7 +598,11 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
       }
       if (!ok) break;
       heap.finish();  // every lane takes part (warp-synchronous flush)
-      if (i_row < Lq) {
+      if (i_row < Lq && parts > 1) {  // this part's kept keys, for the merge
+        const size_t prow = static_cast<size_t>(part) * BH * Lq + static_cast<size_t>(bh) * Lq + i_row;
+        for (int t = 0; t < heap.n; ++t) part_keys[prow * topk + t] = heap.get(t);
+        part_n[prow] = heap.n;
+      } else if (i_row < Lq) {
         const size_t orow = static_cast<size_t>(bh) * Lq + i_row;
         softmax_gather_store<__nv_bfloat16, D>(heap, v + static_cast<size_t>(bh) * Lk * D, out + orow * D);
         if (idx || score)
@@ -582,6 +620,120 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
   }
 }
 
+// Key parts per query tile: split only grids that would leave at least half
+// the SMs idle (a few query tiles against many keys), into as many parts as
+// fill the SMs in one wave, each with at least 4 key tiles.
+int tc_parts(const AttnArgs& a, int num_sms, int N) {
+  const long long units = static_cast<long long>(a.B) * a.H * ((a.Lq + BM - 1) / BM);
+  if (units * 2 > num_sms) return 1;
+  const int kend_min = a.causal ? std::min(a.Lk, BM + (a.Lk - a.Lq)) : a.Lk;  // query tile 0's key range
+  const int nk_min = (kend_min + N - 1) / N;
+  long long p = num_sms / units;
+  p = std::min<long long>(p, nk_min / 4);
+  p = std::min<long long>(p, 8);
+  return static_cast<int>(std::max<long long>(p, 1));
+}
+
+size_t parts_bytes(const AttnArgs& a, int parts) {
+  if (parts <= 1) return 0;
+  const size_t rows = static_cast<size_t>(a.B) * a.H * a.Lq;
+  return static_cast<size_t>(parts) * rows * (static_cast<size_t>(a.topk) * 8 + 4);
+}
+
+constexpr int kMergeWarps = 8;
+
+// Merges a row's `parts` kept lists (each the exact top k of its key range,
+// so the union holds the row's top k): one warp per row sorts the packed keys
+// (descending, a bitonic network in shared memory; empty slots are 0, below
+// every key), keeps the first k, applies the softmax over them and gathers
+// their value rows (each lane D / 32 columns).  Writes the selection too if
+// asked, in the same order as the single-pass kernel.
+template <int D>
+__global__ void __launch_bounds__(kMergeWarps * 32)
+    attn_merge_kernel(const uint64_t* __restrict__ part_keys, const int* __restrict__ part_n, int parts, int BH,
+                      int Lq, int Lk, int topk, int P2, const __nv_bfloat16* __restrict__ v,
+                      __nv_bfloat16* __restrict__ out, int32_t* __restrict__ idx, float* __restrict__ score) {
+  extern __shared__ uint64_t mk_all[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  uint64_t* mk = mk_all + static_cast<size_t>(warp) * P2;
+  const long long rows = static_cast<long long>(BH) * Lq;
+  constexpr int CPL = D / 32;  // columns per lane
+  for (long long r = static_cast<long long>(blockIdx.x) * kMergeWarps + warp; r < rows;
+       r += static_cast<long long>(gridDim.x) * kMergeWarps) {
+    for (int p = 0; p < parts; ++p) {
+      const long long pr = static_cast<long long>(p) * rows + r;
+      // counts and keys are checked before use: after a kernel that stopped
+      // early (a wait ran out) they may never have been written
+      const int n = min(max(__ldg(part_n + pr), 0), topk);
+      for (int t = lane; t < topk; t += 32) {
+        uint64_t key = t < n ? __ldg(reinterpret_cast<const unsigned long long*>(part_keys) + pr * topk + t) : 0ull;
+        if (key_index(key) >= static_cast<uint32_t>(Lk)) key = 0ull;
+        mk[p * topk + t] = key;
+      }
+    }
+    for (int t = parts * topk + lane; t < P2; t += 32) mk[t] = 0ull;
+    __syncwarp();
+    for (int kk = 2; kk <= P2; kk <<= 1)
+      for (int j = kk >> 1; j > 0; j >>= 1) {
+        for (int i = lane; i < P2; i += 32) {
+          const int ixj = i ^ j;
+          if (ixj > i) {
+            const uint64_t x = mk[i], y = mk[ixj];
+            const bool down = (i & kk) == 0;  // this half sorts descending
+            if (down ? (x < y) : (x > y)) {
+              mk[i] = y;
+              mk[ixj] = x;
+            }
+          }
+        }
+        __syncwarp();
+      }
+    int keep = 0;  // nonzero keys sort first
+    for (int t = lane; t < topk; t += 32) keep += mk[t] != 0ull ? 1 : 0;
+    keep = __reduce_add_sync(0xffffffffu, static_cast<unsigned>(keep));
+    const int bh = static_cast<int>(r / Lq);
+    float acc[CPL];
+#pragma unroll
+    for (int e = 0; e < CPL; ++e) acc[e] = 0.f;
+    float z = 0.f;
+    if (keep > 0) {
+      const float m = key_score(mk[0]);
+      const __nv_bfloat16* vb = v + static_cast<size_t>(bh) * Lk * D + lane * CPL;
+      for (int t = 0; t < keep; ++t) {
+        const uint64_t key = mk[t];
+        const float w = expf(key_score(key) - m);
+        z += w;
+        const __nv_bfloat16* vr = vb + static_cast<size_t>(key_index(key)) * D;
+        if constexpr (CPL == 2) {
+          const uint32_t u = __ldg(reinterpret_cast<const unsigned int*>(vr));
+          acc[0] = fmaf(w, __uint_as_float(u << 16), acc[0]);
+          acc[1] = fmaf(w, __uint_as_float(u & 0xffff0000u), acc[1]);
+        } else {
+          const uint2 u = __ldg(reinterpret_cast<const uint2*>(vr));
+          acc[0] = fmaf(w, __uint_as_float(u.x << 16), acc[0]);
+          acc[1] = fmaf(w, __uint_as_float(u.x & 0xffff0000u), acc[1]);
+          acc[2] = fmaf(w, __uint_as_float(u.y << 16), acc[2]);
+          acc[3] = fmaf(w, __uint_as_float(u.y & 0xffff0000u), acc[3]);
+        }
+      }
+    }
+    const float inv = keep > 0 ? 1.f / z : 0.f;
+    __nv_bfloat16* orow = out + static_cast<size_t>(r) * D + lane * CPL;
+#pragma unroll
+    for (int e = 0; e < CPL; e += 2) {
+      __nv_bfloat162 h = __floats2bfloat162_rn(acc[e] * inv, acc[e + 1] * inv);
+      *reinterpret_cast<__nv_bfloat162*>(orow + e) = h;
+    }
+    if (idx || score)
+      for (int t = lane; t < topk; t += 32) {
+        const bool have = t < keep;
+        if (idx) idx[static_cast<size_t>(r) * topk + t] = have ? static_cast<int32_t>(key_index(mk[t])) : -1;
+        if (score) score[static_cast<size_t>(r) * topk + t] = have ? key_score(mk[t]) : -INFINITY;
+      }
+    __syncwarp();
+  }
+}
+
 template <int D, int FK, bool SPLIT>
 int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
   using L = Layout<D, FK, SPLIT>;
@@ -589,7 +741,8 @@ int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t 
   CUtensorMap tmq, tmk;
   if (!make_tmap_bf16_3d(&tmq, a.q, D, a.Lq, BH, BM)) return -1;
   if (!make_tmap_bf16_3d(&tmk, a.k, D, a.Lk, BH, L::N)) return -1;
-  const int n_units = BH * ((a.Lq + BM - 1) / BM);
+  const int parts = tc_parts(a, num_sms, L::N);
+  const int n_units = BH * ((a.Lq + BM - 1) / BM) * parts;
   // At least 120 KB so that a second CTA never shares the SM: each CTA takes
   // all TMEM columns it needs for its whole (persistent) lifetime.
   const size_t need = L::bytes(a.topk);
@@ -599,18 +752,47 @@ int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t 
       cudaSuccess)
     return -1;
   const int grid = n_units < num_sms ? n_units : num_sms;
+  const size_t pbytes = SPLIT ? park_bytes(grid, a.topk) : 0;
+  if (!a.workspace || a.workspace_bytes < pbytes + parts_bytes(a, parts)) {
+    if (SPLIT || parts > 1) return -1;
+  }
+  uint8_t* ws = static_cast<uint8_t*>(a.workspace);
   uint64_t* park = nullptr;
   int* park_n = nullptr;
   if constexpr (SPLIT) {
-    if (!a.workspace || a.workspace_bytes < park_bytes(grid, a.topk)) return -1;
-    park = static_cast<uint64_t*>(a.workspace);
+    park = reinterpret_cast<uint64_t*>(ws);
     park_n = reinterpret_cast<int*>(park + static_cast<size_t>(grid) * park_keys_per_cta(a.topk));
+  }
+  uint64_t* part_keys = nullptr;
+  int* part_n = nullptr;
+  if (parts > 1) {
+    const size_t rows = static_cast<size_t>(BH) * a.Lq;
+    part_keys = reinterpret_cast<uint64_t*>(ws + pbytes);
+    part_n = reinterpret_cast<int*>(part_keys + static_cast<size_t>(parts) * rows * a.topk);
+    // counts start at 0, so that rows a stopped kernel never reached merge as empty
+    if (cudaMemsetAsync(part_n, 0, static_cast<size_t>(parts) * rows * sizeof(int), st) != cudaSuccess) return -1;
   }
   kern<<<grid, kThreads<SPLIT>, smem, st>>>(tmq, tmk, static_cast<const __nv_bfloat16*>(a.v),
                                             static_cast<__nv_bfloat16*>(a.out), BH, a.H, a.Lq, a.Lk, a.topk,
-                                            L::cap(a.topk), a.causal, a.kv_len, n_units, a.idx, a.score, park,
+                                            L::cap(a.topk), a.causal, a.kv_len, n_units, parts, part_keys, part_n,
+                                            parts > 1 ? nullptr : a.idx, parts > 1 ? nullptr : a.score, park,
                                             park_n, ctl);
-  return cudaGetLastError() == cudaSuccess ? 1 : -1;
+  if (cudaGetLastError() != cudaSuccess) return -1;
+  if (parts == 1) return 1;
+  int P2 = 32;
+  while (P2 < parts * a.topk) P2 <<= 1;
+  const size_t msmem = static_cast<size_t>(kMergeWarps) * P2 * 8;
+  auto merge = attn_merge_kernel<D>;
+  if (msmem > 48 * 1024 &&
+      cudaFuncSetAttribute(merge, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(msmem)) != cudaSuccess)
+    return -1;
+  const long long rows = static_cast<long long>(BH) * a.Lq;
+  long long mgrid = (rows + kMergeWarps - 1) / kMergeWarps;
+  if (mgrid > 16LL * num_sms) mgrid = 16LL * num_sms;
+  merge<<<static_cast<unsigned>(mgrid), kMergeWarps * 32, msmem, st>>>(
+      part_keys, part_n, parts, BH, a.Lq, a.Lk, a.topk, P2, static_cast<const __nv_bfloat16*>(a.v),
+      static_cast<__nv_bfloat16*>(a.out), a.idx, a.score);
+  return cudaGetLastError() == cudaSuccess ? 2 : -1;
 }
 
 // Which kernel serves a shape: the split selection where its heaps and rings
@@ -654,11 +836,12 @@ bool attn_tc_supports(const AttnArgs& a) {
 
 size_t attn_tc_workspace_bytes(const AttnArgs& a, int num_sms) {
   if (!attn_tc_supports(a)) return 0;
-  const bool split = a.d == 64 ? is_split(pick<64>(a.topk)) : is_split(pick<128>(a.topk));
-  if (!split) return 0;
-  const long long n_units = static_cast<long long>(a.B) * a.H * ((a.Lq + BM - 1) / BM);
+  const TcKind kind = a.d == 64 ? pick<64>(a.topk) : pick<128>(a.topk);
+  const int N = a.d == 64 ? (is_split(kind) ? TcShape<64, true>::N : TcShape<64, false>::N) : TcShape<128, true>::N;
+  const int parts = tc_parts(a, num_sms, N);
+  const long long n_units = static_cast<long long>(a.B) * a.H * ((a.Lq + BM - 1) / BM) * parts;
   const int grid = n_units < num_sms ? static_cast<int>(n_units) : num_sms;
-  return park_bytes(grid, a.topk);
+  return (is_split(kind) ? park_bytes(grid, a.topk) : 0) + parts_bytes(a, parts);
 }
 
 int attn_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
