@@ -83,7 +83,10 @@ struct Layout {
   using Ring = RingView<BM>;
   static constexpr int N = TcShape<D, SPLIT>::N;
   static constexpr int S = TcShape<D, SPLIT>::S;
-  static constexpr int OW = TcShape<D, SPLIT>::OW;
+  // the two-level heap of 65 <= k <= 137 (up to 137 KB) leaves a row only a
+  // few ring or record slots: one group of 8 per selection call, so that a
+  // call needs one slot (see TcShape<128>)
+  static constexpr int OW = FK == 128 ? 8 : TcShape<D, SPLIT>::OW;
   static constexpr int R = D / 64;  // 128-byte column blocks per row
   static constexpr uint32_t Q_BYTES = BM * D * 2;
   static constexpr uint32_t KST_BYTES = N * D * 2;
@@ -444,13 +447,14 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
           if (lane == 0) mbar_arrive(&acc_empty[b]);
           if (static_cast<int>(jt) + 64 > lim_min) mask_scores(va, jt, lim);
           if (static_cast<int>(jt) + 128 > lim_min) mask_scores(vb, jt + 64u, lim);
+          constexpr int HALF = 64 / OW;  // calls per 64-column half
 #pragma unroll
-          for (int h = 0; h < 4 && ok; ++h) {
+          for (int h = 0; h < 2 * HALF && ok; ++h) {
             if (!f.reserve(OW / 8, ctl, abort_flag)) {
               ok = false;
               break;
             }
-            const float* src = h < 2 ? va + h * OW : vb + (h - 2) * OW;
+            const float* src = h < HALF ? va + h * OW : vb + (h - HALF) * OW;
             f.offer(*reinterpret_cast<const float(*)[OW]>(src), jt + static_cast<uint32_t>(h * OW));
           }
         } else {
@@ -827,10 +831,23 @@ int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st
 
 }  // namespace
 
+// Whether the kernel pick() chooses fits in shared memory.
+template <int D>
+bool tc_fits(int topk) {
+  switch (pick<D>(topk)) {
+    case TcKind::Split64: return Layout<D, 64, true>::fits(topk);
+    case TcKind::Split128: return Layout<D, 128, true>::fits(topk);
+    case TcKind::Split0: return Layout<D, 0, true>::fits(topk);
+    case TcKind::Single64: return Layout<D, 64, false>::fits(topk);
+    case TcKind::Single128: return Layout<D, 128, false>::fits(topk);
+    default: return Layout<D, 0, false>::fits(topk);
+  }
+}
+
 bool attn_tc_supports(const AttnArgs& a) {
   if (a.dtype != 1 || a.topk > kTcMaxK || a.mask) return false;  // bit masks run on the SIMT kernel
-  if (a.d == 64) return Layout<64, 0, false>::fits(a.topk);
-  if (a.d == 128) return Layout<128, 0, false>::fits(a.topk);
+  if (a.d == 64) return tc_fits<64>(a.topk);
+  if (a.d == 128) return tc_fits<128>(a.topk);
   return false;
 }
 
