@@ -133,6 +133,23 @@ int run_attn(const AttnArgs& a, cudaStream_t st) {
   if (!dev) return TOPK_ERR_NO_DEVICE;
   if (dev->cc_major != 10 || dev->cc_minor != 3) return TOPK_ERR_NO_DEVICE;
   const DevCtl ctl = make_ctl(dev);
+  // k at least Lk keeps every valid key (Eq. 4 reduces to Eq. 1): without a
+  // bit mask and without the selection as output, the plain kernel computes it
+  // with no selection at all
+  if (a.topk >= a.Lk && a.dtype == TOPK_BF16 && !a.mask && !a.idx && !a.score &&
+      static_cast<long long>(a.B) * a.H <= 65535) {
+    PlainArgs p{a.q, a.k, a.v, a.out, a.B, a.H, a.Lq, a.Lk, a.d, a.causal, a.kv_len, nullptr};
+    void* pbuf = nullptr;
+    if (!pool_alloc(&pbuf, plain_workspace_bytes(a.B, a.H, a.Lk, a.d), st)) return TOPK_ERR_CUDA;
+    p.workspace = pbuf;
+    const int n = attn_plain(p, ctl, dev->num_sms, st);
+    cudaFreeAsync(pbuf, st);
+    if (n < 0) return TOPK_ERR_CUDA;
+    if (n > 0) {
+      t_last_launches = n;
+      return TOPK_OK;
+    }
+  }
   const size_t ws = attn_tc_workspace_bytes(a, dev->num_sms);
   void* buf = nullptr;
   if (ws && !pool_alloc(&buf, ws, st)) return TOPK_ERR_CUDA;

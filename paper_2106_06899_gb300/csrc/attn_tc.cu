@@ -76,10 +76,15 @@ struct TcShape<128, SPLIT> {
   static constexpr int OW = 8;
 };
 
-template <int D, int FK, bool SPLIT>
+// RPU: query rows per work unit.  The MMA tile always has BM = 128 rows; with
+// RPU = 64 or 32 (single-warp kernel only) just the first RPU of them belong
+// to the unit, so that one row's heap can hold 256 or 512 keys: the heaps of
+// RPU rows of k keys take RPU * k * 8 bytes of shared memory.
+template <int D, int FK, bool SPLIT, int RPU = BM>
 struct Layout {
-  using Sel = RowHeap<BM, FK>;
-  using Heap = HeapCore<BM, FK>;
+  static_assert(RPU == BM || !SPLIT, "reduced-row units run the single-warp kernel");
+  using Sel = RowHeap<RPU, FK>;
+  using Heap = HeapCore<RPU, FK>;
   using Ring = RingView<BM>;
   static constexpr int N = TcShape<D, SPLIT>::N;
   static constexpr int S = TcShape<D, SPLIT>::S;
@@ -191,14 +196,14 @@ __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, const
   }
 }
 
-template <int D, int FK, bool SPLIT>
+template <int D, int FK, bool SPLIT, int RPU = BM>
 __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap tmq, const __grid_constant__ CUtensorMap tmk,
                    const __nv_bfloat16* __restrict__ v, __nv_bfloat16* __restrict__ out, int BH, int H, int Lq,
                    int Lk, int topk, int rec_cap, int causal, const int32_t* __restrict__ kv_len, int n_units,
                    int parts, uint64_t* __restrict__ part_keys, int* __restrict__ part_n, int32_t* __restrict__ idx,
                    float* __restrict__ score, uint64_t* __restrict__ park, int* __restrict__ park_n, DevCtl ctl) {
-  using L = Layout<D, FK, SPLIT>;
+  using L = Layout<D, FK, SPLIT, RPU>;
   using Sel = typename L::Sel;
   constexpr int N = L::N, S = L::S, R = L::R;
   constexpr uint32_t IDESC = idesc_bf16_f32(BM, N);
@@ -253,7 +258,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
 
-  const int n_qt = (Lq + BM - 1) / BM;
+  const int n_qt = (Lq + RPU - 1) / RPU;
   // A unit is (b, h, query tile, key part): with parts > 1 (grids that would
   // leave SMs idle, as decoding a few positions against a long cache does)
   // each query tile's key tiles are split into `parts` ranges, each part keeps
@@ -276,7 +281,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
   const int coff = Lk - Lq;
   auto kv_end = [&](int bh) { return kv_len ? min(max(__ldg(kv_len + bh / H), 0), Lk) : Lk; };
   auto key_tiles = [&](int bh, int qt) {
-    int kend = min(kv_end(bh), causal ? (qt + 1) * BM + coff : Lk);
+    int kend = min(kv_end(bh), causal ? (qt + 1) * RPU + coff : Lk);
     kend = max(kend, 1);
     return (kend + N - 1) / N;
   };
@@ -284,7 +289,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     return static_cast<uint32_t>(min(kv_end(bh), causal ? min(i + 1 + coff, Lk) : Lk));
   };
   auto tile_limit_min = [&](int bh, int qt) {  // the smallest row limit of query tile qt
-    return min(kv_end(bh), causal ? min(qt * BM + 1 + coff, Lk) : Lk);
+    return min(kv_end(bh), causal ? min(qt * RPU + 1 + coff, Lk) : Lk);
   };
   // key tiles [t0, t1) of a unit's part; a part left without tiles streams one
   // fully masked tile (empty = true) so that every stage keeps its handshakes
@@ -316,7 +321,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
       }
       if (lane == 0) {
         mbar_arrive_expect_tx(q_full, L::Q_BYTES);
-        for (int r = 0; r < R; ++r) tma_load_3d(q_s + r * BM * 128, &tmq, q_full, r * 64, qt * BM, bh);
+        for (int r = 0; r < R; ++r) tma_load_3d(q_s + r * BM * 128, &tmq, q_full, r * 64, qt * RPU, bh);
       }
       ++q_issued;
       int t0, t1;
@@ -558,6 +563,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     // ------------------------------------------------------------ selection
     const int quad = warp & 3;
     const int row = quad * 32 + lane;
+    const bool active = quad < RPU / 32;  // lanes of the MMA tile that belong to the unit
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
     uint32_t acc_it = 0;
     Sel heap;
@@ -565,8 +571,8 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
     for (int u = blockIdx.x; ok && u < n_units; u += gridDim.x) {
       int bh, qt, part;
       decode(u, bh, qt, part);
-      const int i_row = qt * BM + row;
-      heap.init(sel_mem, row, topk, rec_cap);
+      const int i_row = qt * RPU + row;
+      if (active) heap.init(sel_mem, row, topk, rec_cap);
       int t0, t1;
       bool empty;
       tile_range(bh, qt, part, t0, t1, empty);
@@ -579,6 +585,12 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
           break;
         }
         tc_fence_after();
+        if (!active) {  // no rows of this unit in these lanes: release the accumulator
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&acc_empty[b]);
+          continue;
+        }
         const uint32_t taddr = tmem_base + lane_base + static_cast<uint32_t>(b * N);
         const uint32_t jt = static_cast<uint32_t>(kt * N);
 #pragma unroll 1
@@ -601,6 +613,7 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
         }
       }
       if (!ok) break;
+      if (!active) continue;
       heap.finish();  // every lane takes part (warp-synchronous flush)
       if (i_row < Lq && parts > 1) {  // this part's kept keys, for the merge
         const size_t prow = static_cast<size_t>(part) * BH * Lq + static_cast<size_t>(bh) * Lq + i_row;
@@ -627,10 +640,10 @@ __global__ void __launch_bounds__(kThreads<SPLIT>, 1)
 // Key parts per query tile: split only grids that would leave at least half
 // the SMs idle (a few query tiles against many keys), into as many parts as
 // fill the SMs in one wave, each with at least 4 key tiles.
-int tc_parts(const AttnArgs& a, int num_sms, int N) {
-  const long long units = static_cast<long long>(a.B) * a.H * ((a.Lq + BM - 1) / BM);
+int tc_parts(const AttnArgs& a, int num_sms, int N, int rpu) {
+  const long long units = static_cast<long long>(a.B) * a.H * ((a.Lq + rpu - 1) / rpu);
   if (units * 2 > num_sms) return 1;
-  const int kend_min = a.causal ? std::min(a.Lk, BM + (a.Lk - a.Lq)) : a.Lk;  // query tile 0's key range
+  const int kend_min = a.causal ? std::min(a.Lk, rpu + (a.Lk - a.Lq)) : a.Lk;  // query tile 0's key range
   const int nk_min = (kend_min + N - 1) / N;
   long long p = num_sms / units;
   p = std::min<long long>(p, nk_min / 4);
@@ -738,20 +751,20 @@ __global__ void __launch_bounds__(kMergeWarps * 32)
   }
 }
 
-template <int D, int FK, bool SPLIT>
+template <int D, int FK, bool SPLIT, int RPU = BM>
 int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st) {
-  using L = Layout<D, FK, SPLIT>;
+  using L = Layout<D, FK, SPLIT, RPU>;
   const int BH = a.B * a.H;
   CUtensorMap tmq, tmk;
   if (!make_tmap_bf16_3d(&tmq, a.q, D, a.Lq, BH, BM)) return -1;
   if (!make_tmap_bf16_3d(&tmk, a.k, D, a.Lk, BH, L::N)) return -1;
-  const int parts = tc_parts(a, num_sms, L::N);
-  const int n_units = BH * ((a.Lq + BM - 1) / BM) * parts;
+  const int parts = tc_parts(a, num_sms, L::N, RPU);
+  const int n_units = BH * ((a.Lq + RPU - 1) / RPU) * parts;
   // At least 120 KB so that a second CTA never shares the SM: each CTA takes
   // all TMEM columns it needs for its whole (persistent) lifetime.
   const size_t need = L::bytes(a.topk);
   const size_t smem = need > 120 * 1024 ? need : 120 * 1024;
-  auto kern = attn_tc_kernel<D, FK, SPLIT>;
+  auto kern = attn_tc_kernel<D, FK, SPLIT, RPU>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
       cudaSuccess)
     return -1;
@@ -802,7 +815,9 @@ int launch_tc_k(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t 
 // Which kernel serves a shape: the split selection where its heaps and rings
 // fit, else the single-warp kernel; fixed heap shapes: 8-ary for k = 64,
 // two-level (8 x 16) for 65 <= k <= 137.
-enum class TcKind { Split64, Split128, Split0, Single64, Single128, Single0 };
+// and, for k above what 128 rows' heaps can hold, the single-warp kernel on
+// units of 64 (k <= 256) or 32 (k <= 512) query rows.
+enum class TcKind { Split64, Split128, Split0, Single64, Single128, Single0, Single0R64, Single0R32 };
 
 template <int D>
 TcKind pick(int topk) {
@@ -812,8 +827,12 @@ TcKind pick(int topk) {
   if (Layout<D, 0, true>::fits(topk)) return TcKind::Split0;
   if (topk == 64 && Layout<D, 64, false>::fits(64)) return TcKind::Single64;
   if (two_level && Layout<D, 128, false>::fits(topk)) return TcKind::Single128;
-  return TcKind::Single0;
+  if (Layout<D, 0, false>::fits(topk)) return TcKind::Single0;
+  if (topk <= 256 && Layout<D, 0, false, 64>::fits(topk)) return TcKind::Single0R64;
+  return TcKind::Single0R32;
 }
+
+int rows_per_unit(TcKind k) { return k == TcKind::Single0R64 ? 64 : (k == TcKind::Single0R32 ? 32 : BM); }
 
 bool is_split(TcKind k) { return k == TcKind::Split64 || k == TcKind::Split128 || k == TcKind::Split0; }
 
@@ -825,6 +844,8 @@ int launch_tc(const AttnArgs& a, const DevCtl& ctl, int num_sms, cudaStream_t st
     case TcKind::Split0: return launch_tc_k<D, 0, true>(a, ctl, num_sms, st);
     case TcKind::Single64: return launch_tc_k<D, 64, false>(a, ctl, num_sms, st);
     case TcKind::Single128: return launch_tc_k<D, 128, false>(a, ctl, num_sms, st);
+    case TcKind::Single0R64: return launch_tc_k<D, 0, false, 64>(a, ctl, num_sms, st);
+    case TcKind::Single0R32: return launch_tc_k<D, 0, false, 32>(a, ctl, num_sms, st);
     default: return launch_tc_k<D, 0, false>(a, ctl, num_sms, st);
   }
 }
@@ -840,6 +861,8 @@ bool tc_fits(int topk) {
     case TcKind::Split0: return Layout<D, 0, true>::fits(topk);
     case TcKind::Single64: return Layout<D, 64, false>::fits(topk);
     case TcKind::Single128: return Layout<D, 128, false>::fits(topk);
+    case TcKind::Single0R64: return Layout<D, 0, false, 64>::fits(topk);
+    case TcKind::Single0R32: return Layout<D, 0, false, 32>::fits(topk);
     default: return Layout<D, 0, false>::fits(topk);
   }
 }
@@ -855,8 +878,9 @@ size_t attn_tc_workspace_bytes(const AttnArgs& a, int num_sms) {
   if (!attn_tc_supports(a)) return 0;
   const TcKind kind = a.d == 64 ? pick<64>(a.topk) : pick<128>(a.topk);
   const int N = a.d == 64 ? (is_split(kind) ? TcShape<64, true>::N : TcShape<64, false>::N) : TcShape<128, true>::N;
-  const int parts = tc_parts(a, num_sms, N);
-  const long long n_units = static_cast<long long>(a.B) * a.H * ((a.Lq + BM - 1) / BM) * parts;
+  const int rpu = rows_per_unit(kind);
+  const int parts = tc_parts(a, num_sms, N, rpu);
+  const long long n_units = static_cast<long long>(a.B) * a.H * ((a.Lq + rpu - 1) / rpu) * parts;
   const int grid = n_units < num_sms ? static_cast<int>(n_units) : num_sms;
   return (is_split(kind) ? park_bytes(grid, a.topk) : 0) + parts_bytes(a, parts);
 }

@@ -14,8 +14,9 @@ namespace topk {
 // topk x rows x 8 bytes of shared memory).
 constexpr int kSimtSmallRowsMaxK = 128;
 constexpr int kSimtMaxK = 512;
-// tcgen05 attention path limit (heap for 128 rows in shared memory)
-constexpr int kTcMaxK = 128;
+// tcgen05 attention path limit: 128 rows' heaps up to k = 137, units of 64 or
+// 32 query rows up to 256 or 512 (heaps in shared memory)
+constexpr int kTcMaxK = 512;
 
 struct AttnArgs {
   const void* q;
