@@ -280,3 +280,17 @@ def test_ragged_long_rows(d, topk):
     # 128-row tile, several heads
     q, k, v = W.attention_inputs(1, 3, 300, 33000 + d, d, dtype="bf16", seed=600 + topk + d)
     _check(q, k, v, topk, "bf16")
+
+
+@pytest.mark.parametrize("d,k,causal", [(64, 256, False), (64, 512, True), (128, 160, True)])
+def test_reduced_row_units_sampled(d, k, causal):
+    # 64- and 32-row units at a longer sequence, with the selection output (no plain-kernel shortcut)
+    B, H, L = 1, 3, 3000
+    q, kk, v = W.attention_inputs(B, H, L, L, d, seed=400 + k)
+    rows = W.sample_rows(B * H * L, 300, seed=k).numpy()
+    out, idx, score = T.attention(q.cuda(), kk.cuda(), v.cuda(), k, causal=causal, return_indices=True)
+    T.topk_check()
+    st = check_rows(q=q, k=kk, v=v, rows=rows, gpu_out=out.float().reshape(-1, d).cpu().numpy()[rows],
+                    gpu_idx=idx.reshape(-1, k).cpu().numpy()[rows], gpu_score=score.reshape(-1, k).cpu().numpy()[rows],
+                    topk=k, dtype="bf16", causal=causal)
+    assert st["exact_set_frac"] > 0.95, st

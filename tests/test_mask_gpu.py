@@ -117,3 +117,13 @@ def test_masked_forward_then_backward():
     for name, g, r in pairs:
         assert np.abs(g - r).max() <= 2e-5 * np.abs(r).max() + 1e-30, name
     assert not dk.cpu()[1, :, 300:].any() and not dv.cpu()[1, :, 300:].any()
+
+
+@pytest.mark.parametrize("d,k", [(64, 200), (128, 300)])
+def test_masks_on_reduced_row_units(d, k):
+    # k above 137 runs on 64- or 32-row units: causal decode, key counts and key parts together
+    B, H, Lq, Lk = 2, 2, 70, 1500
+    q, kk, v = W.attention_inputs(B, H, Lq, Lk, d, seed=93)
+    st, out, idx = _check(q, kk, v, k, causal=True, kv_len=[1500, 180])
+    assert torch.all((idx[1] >= 0).sum(-1) == 180)  # every row of batch 1 keeps all its 180 keys
+    assert st["exact_set_frac"] > 0.95, st
