@@ -220,6 +220,37 @@ struct HeapCore {
     return act ? top : cur;
   }
 
+  // Branch-free root replacement in a full 4-ary heap (FIXED_K == 0) of at
+  // most 1364 keys: if act, x (which must rank above the root) replaces the
+  // root.  Five levels are always walked with predicated stores, and a child
+  // past k reads as the largest key, so lanes that disagree on act or on the
+  // depth run one straight-line body.  Returns the root after the call (cur
+  // when act is false).
+  __device__ __forceinline__ uint64_t replace_pred4(uint64_t x, bool act, uint64_t cur) {
+    int p = 0;
+    bool go = act;
+    uint64_t top = x;
+#pragma unroll
+    for (int level = 0; level < 5; ++level) {
+      const int c = 4 * p + 1;
+      uint64_t ch[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) ch[q] = c + q < k ? get(c + q) : ~0ull;
+      const bool l01 = ch[0] <= ch[1], l23 = ch[2] <= ch[3];
+      const uint64_t m01 = l01 ? ch[0] : ch[1], m23 = l23 ? ch[2] : ch[3];
+      const int i01 = l01 ? 0 : 1, i23 = l23 ? 2 : 3;
+      const bool lf = m01 <= m23;
+      const uint64_t a = lf ? m01 : m23;
+      const bool down = go && a < x;
+      if (level == 0) top = down ? a : x;
+      st_shared_u64_if(go, base + p * ROWS, down ? a : x);  // the child moves up, or x settles here
+      p = down ? c + (lf ? i01 : i23) : p;
+      go = down;
+    }
+    st_shared_u64_if(go, base + p * ROWS, x);  // below the fifth level
+    return act ? top : cur;
+  }
+
   // Smallest of NC keys (a power of two) and its first position (a tree).
   template <int NC>
   __device__ __forceinline__ static void argmin_n(const uint64_t (&ch)[NC], uint64_t& m, int& i) {
@@ -452,9 +483,26 @@ struct RowHeap : HeapCore<ROWS, FIXED_K> {
     float x = -INFINITY;
     uint32_t j = 0;
     if (cnt > 0) fetch(0, x, j);
-    bool fast = false;
-    if constexpr (FIXED_K == 64 || FIXED_K == 128) fast = __all_sync(0xffffffffu, Core::n == Core::k);
-    if (fast) {
+    const bool fast = __all_sync(0xffffffffu, Core::n == Core::k);
+    if constexpr (FIXED_K == 0) {
+      if (fast) {  // every heap is full: one straight-line 4-ary replace per step
+        uint64_t r = Core::root;
+        for (int t = 0; t < mx; ++t) {
+          float xn = -INFINITY;
+          uint32_t jn = 0;
+          if (t + 1 < cnt) fetch(t + 1, xn, jn);
+          const uint64_t key = make_key(x, j);
+          r = Core::replace_pred4(key, t < cnt && key > r, r);
+          x = xn;
+          j = jn;
+        }
+        Core::root = r;
+        tau = key_score(r);
+        rc = 0;
+        return;
+      }
+    }
+    if (FIXED_K != 0 && fast) {
       // every heap is full: one straight-line replace per step, the root and
       // its 8 children in registers, written back once
       uint64_t r = Core::root;
@@ -761,9 +809,18 @@ struct RowSink : HeapCore<ROWS, FIXED_K> {
     st_release_u32(v.tail, t);
     const int mx = __reduce_max_sync(0xffffffffu, static_cast<unsigned>(cnt));
     uint2 c = cnt > 0 ? v.stage[0] : make_uint2(0u, 0u);
-    bool fast = false;
-    if constexpr (FIXED_K == 64 || FIXED_K == 128) fast = __all_sync(0xffffffffu, n == k);
-    if (fast) {
+    const bool fast = __all_sync(0xffffffffu, n == k);
+    if (FIXED_K == 0 && fast) {  // every kept set is full: one straight-line 4-ary replace per step
+      uint64_t r = Core::root;
+      for (int q = 0; q < mx; ++q) {
+        const uint2 cn = q + 1 < cnt ? v.stage[(q + 1) * ROWS] : make_uint2(0u, 0u);
+        const uint64_t key = make_key(__uint_as_float(c.x), c.y);
+        r = Core::replace_pred4(key, q < cnt && key > r, r);
+        c = cn;
+      }
+      Core::root = r;
+      tau = key_score(r);
+    } else if (FIXED_K != 0 && fast) {
       // every kept set is full: one straight-line replace per step
       uint64_t r = Core::root;
       uint64_t ch0[8];
