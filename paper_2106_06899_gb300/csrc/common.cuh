@@ -70,10 +70,12 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 
 // Waits until the phase with the given parity has completed.  Returns false
 // (after flagging the error and the CTA abort word) if the limit runs out or
-// another thread of the CTA already gave up.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const DevCtl& ctl,
-                                          volatile int* abort_flag) {
-  if (mbar_try_wait(bar, parity)) return true;
+// another thread of the CTA already gave up.  The polling loop is out of line
+// (mbar_wait_slow): each wait site holds one try and a call instead of the
+// loop, which keeps the kernels' unrolled pipelines small in the instruction
+// cache.
+static __device__ __noinline__ bool mbar_wait_slow(uint64_t* bar, uint32_t parity, const DevCtl& ctl,
+                                                   volatile int* abort_flag) {
   const unsigned long long t0 = global_ns();
   for (uint32_t spin = 1;; ++spin) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -86,6 +88,12 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const 
       }
     }
   }
+}
+
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, const DevCtl& ctl,
+                                          volatile int* abort_flag) {
+  if (mbar_try_wait(bar, parity)) return true;
+  return mbar_wait_slow(bar, parity, ctl, abort_flag);
 }
 
 // ---------------------------------------------------------------- CTA-scope
