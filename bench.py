@@ -149,14 +149,17 @@ def work_flops(w) -> float:
     return 2.0 * w.B * w.H * w.Lq * w.Lk * w.d
 
 
+# the largest k of the bf16 tensor-core attention kernels (kTcMaxK of the library)
+TC_MAX_K = 512
+
 # fp32 FMA rate of the CUDA cores: 152 SMs x 128 fp32 lanes x 2 FLOP x 2.07 GHz (maximum SM clock)
 FP32_FMA_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 
 
 def roofline(w, achieved, pk):
     """Roofline of the dominant kernel: the tcgen05 kernels against the measured bf16 tensor peak; the
-    SIMT kernel (fp32 inputs, or k above the tensor path's 128) against the fp32 FMA rate."""
-    simt = w.kind == "attn" and (w.dtype == "f32" or w.topk > 128 or w.mask_p > 0)
+    SIMT kernel (fp32 inputs, a bit mask, or k above the tensor path's 512) against the fp32 FMA rate."""
+    simt = w.kind == "attn" and (w.dtype == "f32" or w.topk > TC_MAX_K or w.mask_p > 0)
     if simt:
         return {"bound": "alu", "achieved": achieved, "peak": FP32_FMA_TFLOPS, "unit": "TFLOP/s",
                 "frac": achieved / FP32_FMA_TFLOPS, "traffic": None,
