@@ -747,8 +747,9 @@ def run_plain(args):
         ref = oracle.ffn_dense(*host, rows=rows)
         t = time.perf_counter() - t0
         got = out.cpu().numpy()[rows]
-        # H = ReLU(x W1^T) is rounded to bf16 before the second product: an element may be off by
-        # 2^-9 sum_j H_j |W2_j| (the dense layer on |W2|) plus the fp32 sums
+        # H = ReLU(x W1^T) is rounded to bf16 (relative error at most 2^-8) before the second
+        # product: an element may be off by 2^-8 sum_j H_j |W2_j| (the dense layer on |W2|) plus
+        # the fp32 sums
         bound = 2.0 ** -8 * oracle.ffn_dense(host[0], host[1], host[2].abs(), rows=rows) + 1e-5
     else:
         okv, _ = oracle_masks(w.with_(mask_p=0.0))
