@@ -47,8 +47,10 @@
  *     stream-ordered memory pool that the library owns (one per device) and
  *     returned to it on `stream`; its size is reported by the
  *     *_workspace_bytes queries and is never proportional to Lq * Lk: a
- *     fixed amount per SM for attention, linear in the tokens for the
- *     feed-forward layer.  The pool keeps returned memory
+ *     fixed amount per SM for attention (plus, when a grid of few query
+ *     tiles is split into key parts, each part's kept list per row), linear
+ *     in the tokens for the feed-forward layer and in the cache for the
+ *     backward calls.  The pool keeps returned memory
  *     reserved for later calls (up to the largest amount in use at once),
  *     so that repeated calls do not map device memory again each time, until
  *     topk_pool_trim() hands it back or the process exits;
@@ -96,7 +98,9 @@ enum {
  *   topk         : 1 <= topk <= Lk; the supported maximum is 512.
  *   chunk        : query-chunk size (Sec. 2.2), >= 1; a scheduling hint only.
  *   causal       : 0 or 1.
- *   Scratch: topk_attn_workspace_bytes() (a fixed amount per SM, or none).
+ *   Scratch: topk_attn_workspace_bytes() (a fixed amount per SM, or none;
+ *            plus parts x B*H*Lq x (8 topk + 4) bytes where at most half the
+ *            SMs would get a query tile and the key tiles are split into parts).
  * Errors: TOPK_ERR_INVALID_ARG / TOPK_ERR_UNSUPPORTED before any launch;
  *         TOPK_ERR_CUDA if a launch fails (or the scratch cannot be had).
  *         A device-side timeout is not returned by this call (it returns
